@@ -1,0 +1,44 @@
+"""Planted mistakes in the oracle (on the CPU only) must each fail some pin.
+
+Every mutation below is a plausible slip in writing the method down: a causal
+mask, a wrong softmax scale, interleaved instead of contiguous GQA groups, the
+last instead of the first maximum, a strict threshold, ties broken towards the
+higher index, a rounded-up remask count. If a pin suite let one through, the
+oracle could carry that slip undetected."""
+import math
+
+import numpy as np
+import pytest
+
+import oracle_pins as P
+from oracle import attention as oatt
+from oracle import update as oupd
+from oracle import vocab as ovoc
+
+MUTATIONS = {
+    "causal_mask": (oatt, "key_mask", lambda n: np.tril(np.ones((n, n), dtype=bool)), P.ATTN_PINS),
+    "scale_1_over_D": (oatt, "score_scale", lambda D: 1.0 / D, P.ATTN_PINS),
+    "interleaved_gqa": (oatt, "kv_head", lambda h, Hq, Hkv: h % Hkv, P.ATTN_PINS),
+    "last_argmax": (ovoc, "first_argmax",
+                    lambda x: x.shape[1] - 1 - np.argmax(x[:, ::-1], axis=1), P.VOCAB_PINS),
+    "strict_threshold": (oupd, "is_edit", lambda p, t, c, tau: p != t and c > tau, P.UPDATE_PINS),
+    "ties_high_index": (oupd, "remask_order",
+                        lambda cv, pos: sorted(pos, key=lambda i: (cv[i], -i)), P.UPDATE_PINS),
+    "ceil_remask_count": (oupd, "remask_count",
+                          lambda k, f, r: max(0, min(k if k >= 0 else
+                                                     math.ceil(float(np.float32(f)) * r), r)),
+                          P.UPDATE_PINS),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_mutation_is_caught(name, monkeypatch):
+    mod, attr, fn, pins = MUTATIONS[name]
+    monkeypatch.setattr(mod, attr, fn)
+    failed = []
+    for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            failed.append(pin.__name__)
+    assert failed, f"mutation {name} passed every pin"
