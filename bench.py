@@ -1,0 +1,462 @@
+"""Throughput of one bidirectional refine step (attention -> vocabulary
+reduction -> update) on GB300, as refine steps/s over a whole batch.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+Default workload: the batched 32 x 512 refine (128 prompt + 384 response
+tokens per sequence, prompts U{64..256}, 32/4 heads, head_dim 128,
+V = 151552, bf16). Inputs are synthetic (seeded generator) and resident in HBM
+before timing; every input is larger than L2, so no flush is needed.
+
+Prints one JSON line (rank 0). For N > 1 (torchrun) every rank runs its own
+replica on its own seeded batch (weak scaling, no collective on the data
+path); the step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "refine_steps_per_sec"
+UNIT = "steps/s"
+DEFAULT_CONFIG = "c3_batch32_512"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return {"hbm_gbs": pk["hbm_gbs"], "bf16_tflops": pk["bf16_tflops"],
+                "bf16_tflops_sustained": pk.get("bf16_tflops_sustained"), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """Samples nvidia-smi SM clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- traffic record
+
+def kernel_source_sha(fname: str) -> str:
+    h = hashlib.sha256()
+    for f in (fname, "dlm_common.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_02625_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel_file: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source
+    still matches the one profiled (else None)."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)
+        e = rec[kernel_file][workload]
+        if e["source_sha"] != kernel_source_sha(kernel_file):
+            return None
+        return e["dram_bytes_per_launch"]
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------------- CPU oracle timing
+
+def _oracle_worker(conn, name, b, vocab_rows):
+    """A host core timing the oracle on sequence b of the workload: fp64
+    attention over every head, the vocabulary reduction of `vocab_rows` of its
+    rows (spread over the sequence), and the update of the whole sequence.
+    Inputs are generated once, before any timing."""
+    import numpy as np
+    import oracle
+    from paper_2608_02625_gb300 import synth, workloads
+    w = workloads.get(name)
+
+    def host(which, H):
+        per = w.L * H * w.D
+        x = synth.qkv_host(w.seed, which, (w.B, w.L, H, w.D), w.qkv_sigma, w.dtype, b * per, per)
+        x = synth.bf16_bits_to_f32(x) if w.dtype == "bf16" else x
+        return x.reshape(1, w.L, H, w.D)
+
+    q, k, v = host(synth.S_Q, w.Hq), host(synth.S_K, w.Hkv), host(synth.S_V, w.Hkv)
+    tok, msk = w.initial_state()
+    rows = b * w.L + np.linspace(0, w.L - 1, vocab_rows).astype(np.int64)
+    x = w.logit_spec(0).rows_f32(rows, tok.reshape(-1)[rows], msk.reshape(-1)[rows])
+    if w.dtype == "bf16":
+        x = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(x))
+    # The update reads a full sequence of predictions; the sampled rows' values
+    # are tiled over it (the update's cost does not depend on the values).
+    reps = -(-w.L // vocab_rows)
+    n, p = w.seq_lens()[b:b + 1], w.prompt_lens()[b:b + 1]
+    conn.send("ready")
+    while conn.recv() == "run":
+        t0 = time.perf_counter()
+        oracle.bidir_attn(q, k, v, n)
+        t1 = time.perf_counter()
+        am, cf, _ = oracle.vocab_confidence(x)
+        t2 = time.perf_counter()
+        oracle.refine_update(tok[b:b + 1], msk[b:b + 1], np.tile(am, reps)[None, :w.L],
+                             np.tile(cf, reps)[None, :w.L], edit_threshold=w.edit_threshold[0],
+                             remask_k=w.remask_k, remask_frac=w.remask_frac, mask_id=w.mask_id,
+                             prompt_lens=p, seq_lens=n)
+        t3 = time.perf_counter()
+        conn.send((t1 - t0, (t2 - t1) * w.L / vocab_rows, t3 - t2))
+
+
+class OracleTimer:
+    """`workers` single-threaded processes (spawned), one sequence each."""
+
+    VOCAB_ROWS = 64
+
+    def __init__(self, name: str, workers: int):
+        from paper_2608_02625_gb300 import workloads
+        self.w = workloads.get(name)
+        self.name = name
+        os.environ["OPENBLAS_NUM_THREADS"] = "1"
+        os.environ["OMP_NUM_THREADS"] = "1"
+        ctx = mp.get_context("spawn")
+        self.conns, self.procs = [], []
+        for i in range(workers):
+            a, bconn = ctx.Pipe()
+            pr = ctx.Process(target=_oracle_worker, args=(bconn, name, (i * 7) % self.w.B, self.VOCAB_ROWS),
+                             daemon=True)
+            pr.start()
+            self.conns.append(a)
+            self.procs.append(pr)
+        self.ready = False
+
+    def _wait_ready(self):
+        if not self.ready:
+            for c in self.conns:
+                assert c.recv() == "ready"
+            self.ready = True
+
+    def run(self):
+        """One round: every worker times its sequence. Returns cpu_baseline."""
+        self._wait_ready()
+        for c in self.conns:
+            c.send("run")
+        parts = [c.recv() for c in self.conns]
+        per_seq = [sum(x) for x in parts]
+        mean_seq = statistics.mean(per_seq)
+        w = self.w
+        cores = len(self.conns)
+        return {"value": cores / (mean_seq * w.B), "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": (f"{cores} of the {w.B} sequences of {self.name}, one per single-threaded process: "
+                           f"fp64 attention over all {w.Hq} heads, vocabulary reduction of {self.VOCAB_ROWS} of "
+                           f"its {w.L} rows scaled to {w.L}, update of the whole sequence; "
+                           f"steps/s = cores / (B x mean seconds per sequence)"),
+                "oracle_s_per_sequence": {"attn": statistics.mean(x[0] for x in parts),
+                                          "vocab": statistics.mean(x[1] for x in parts),
+                                          "update": statistics.mean(x[2] for x in parts)}}
+
+    def close(self):
+        for c in self.conns:
+            try:
+                c.send("stop")
+            except Exception:
+                pass
+        for pr in self.procs:
+            pr.join(timeout=10)
+
+
+def host_workers():
+    return max(1, min(16, (os.cpu_count() or 2) - 1))
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def run_ours(args, rank, world):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_02625_gb300 import binding as Bn
+    from paper_2608_02625_gb300 import synth_gpu, workloads
+
+    base = workloads.get(args.config)
+    # Weak scaling: each rank refines its own seeded batch of the same shape.
+    w = workloads.scaled(base, seed=base.seed + rank)
+    d = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(d)
+    peaks = load_peaks()
+
+    timer = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        timer = OracleTimer(base.name, host_workers())   # spawned before any GPU work
+
+    # Inputs resident in HBM.
+    q, k, v = synth_gpu.qkv(w, 0, d)
+    tok_np, msk_np = w.initial_state()
+    tok = torch.from_numpy(tok_np).to(d)
+    msk = torch.from_numpy(msk_np).to(d)
+    logits = synth_gpu.logits(w, 0, d, tok.view(-1), msk.view(-1))
+    prompt = torch.from_numpy(w.prompt_lens()).to(d)
+    seqlen = torch.from_numpy(w.seq_lens()).to(d)
+    out = torch.empty_like(q)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
+    stream = torch.cuda.current_stream(d)
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+        if ev:
+            ev[1].record(stream)
+        Bn.dlm_vocab_confidence(logits, am, cf, ls)
+        if ev:
+            ev[2].record(stream)
+        Bn.dlm_refine_update(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), params, nt, nm, ne)
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during warm-up")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(d.index if d.index is not None else 0) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    per_kernel = {
+        "attn": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
+        "vocab": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
+        "update": statistics.mean(e[2].elapsed_time(e[3]) for e in evs),
+    }
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the timed region")
+    t = torch.tensor([total_ms], dtype=torch.float64, device=d)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        h_q, h_k, h_v = q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory()
+        h_logits = torch.empty(logits.shape, dtype=logits.dtype, pin_memory=True)
+        h_logits.copy_(logits)
+        h_tok, h_msk = tok.cpu().pin_memory(), msk.cpu().pin_memory()
+        h_p, h_n = prompt.cpu().pin_memory(), seqlen.cpu().pin_memory()
+        o_tok = torch.empty(tok.shape, dtype=tok.dtype, pin_memory=True)
+        o_msk = torch.empty(msk.shape, dtype=msk.dtype, pin_memory=True)
+        o_ne = torch.empty(ne.shape, dtype=ne.dtype, pin_memory=True)
+        ins = [(h_q, q), (h_k, k), (h_v, v), (h_logits, logits), (h_tok, tok), (h_msk, msk), (h_p, prompt),
+               (h_n, seqlen)]
+        outs = [(nt, o_tok), (nm, o_msk), (ne, o_ne)]
+        h2d = sum(h.numel() * h.element_size() for h, _ in ins)
+        d2h = sum(h.numel() * h.element_size() for _, h in outs)
+
+        def e2e_step():
+            for h, dv in ins:
+                dv.copy_(h, non_blocking=True)
+            step()
+            for dv, h in outs:
+                h.copy_(dv, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        k_e2e = max(2, min(args.steps, 10))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(k_e2e):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        te = torch.tensor([e0.elapsed_time(e1) / k_e2e], dtype=torch.float64, device=d)
+        if world > 1:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e2e = {"value": world * 1000.0 / float(te.item()), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": float(te.item()), "steps": k_e2e}
+
+    if rank != 0:
+        return None
+
+    attn_flops = w.attn_flops()
+    vocab_bytes = w.vocab_bytes()
+    kern = {
+        "attn": {"achieved_tflops": attn_flops / (per_kernel["attn"] * 1e-3) / 1e12, "ms": per_kernel["attn"],
+                 "flops": attn_flops},
+        "vocab": {"achieved_gbs": vocab_bytes / (per_kernel["vocab"] * 1e-3) / 1e9, "ms": per_kernel["vocab"],
+                  "bytes": vocab_bytes},
+        "update": {"ms": per_kernel["update"]},
+    }
+    kern["attn"]["frac_of_measured_bf16"] = kern["attn"]["achieved_tflops"] / peaks["bf16_tflops"]
+    kern["vocab"]["frac_of_measured_hbm"] = kern["vocab"]["achieved_gbs"] / peaks["hbm_gbs"]
+    dominant = max(("attn", "vocab"), key=lambda kk: per_kernel[kk])
+    if dominant == "vocab":
+        roof = {"kernel": "vocab_confidence", "bound": "hbm", "achieved": kern["vocab"]["achieved_gbs"],
+                "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": kern["vocab"]["frac_of_measured_hbm"],
+                "traffic": recorded_traffic("vocab.cu", base.name), "algorithmic_bytes": vocab_bytes,
+                "peak_source": peaks["source"]}
+    else:
+        roof = {"kernel": "bidir_attn", "bound": "tensor", "achieved": kern["attn"]["achieved_tflops"],
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s", "frac": kern["attn"]["frac_of_measured_bf16"],
+                "traffic": recorded_traffic("attn_tc.cu", base.name), "algorithmic_flops": attn_flops,
+                "peak_source": peaks["source"]}
+
+    steps_per_s = world * 1000.0 / ms_per_step
+    res = {
+        "metric": METRIC, "value": steps_per_s, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded counter-based generator, resident in HBM)",
+        "config": {"workload": base.name, "batch": w.B, "seq_len": w.L, "q_heads": w.Hq, "kv_heads": w.Hkv,
+                   "head_dim": w.D, "vocab": w.V, "refined_tokens_per_step": w.refined_tokens(),
+                   "l2": "no flush: logits and q/k/v are larger than L2 (129 MB)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "refined_tokens_per_sec": steps_per_s * w.refined_tokens(),
+        "kernels": kern,
+        "roofline": roof,
+        "gpu_launches": 3 * args.steps,
+        "e2e": e2e,
+    }
+    if timer is not None:
+        res["cpu_baseline"] = timer.run()
+        timer.close()
+    res["clocks"] = clk.summary()
+    res["peaks"] = peaks
+    return res
+
+
+def run_reference(args, rank, world):
+    """The oracle as the reference arm: each step is one round of the host
+    cores timing their sample of the same workload, scaled to steps/s."""
+    if rank != 0:
+        return None
+    timer = OracleTimer(args.config, host_workers())
+    for _ in range(args.warmup):
+        timer.run()
+    vals = [timer.run() for _ in range(args.steps)]
+    timer.close()
+    value = statistics.mean(v["value"] for v in vals)
+    from paper_2608_02625_gb300 import workloads
+    w = workloads.get(args.config)
+    cb = dict(vals[-1])
+    cb["value"] = value
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "batch": w.B, "seq_len": w.L, "q_heads": w.Hq, "kv_heads": w.Hkv,
+                       "head_dim": w.D, "vocab": w.V},
+            "refined_tokens_per_sec": value * w.refined_tokens(),
+            "cpu_baseline": cb, "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                                        "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist.init_process_group("nccl")
+    res = run_reference(args, rank, world) if args.impl == "reference" else run_ours(args, rank, world)
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

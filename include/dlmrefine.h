@@ -1,0 +1,184 @@
+/*
+ * libdlmrefine -- one bidirectional refine step of speculative correction
+ * (draft-then-refine decoding for diffusion language models), on GB300.
+ *
+ * The refiner receives the fixed prompt plus a complete draft and revises any
+ * response position with full-sequence bidirectional denoising passes
+ * (Sec. 4.2). One pass on the hot path is three calls, in this order:
+ *
+ *   dlm_bidir_attn        non-causal GQA attention over all valid positions
+ *   dlm_vocab_confidence  per position: argmax token, max softmax probability,
+ *                         log-sum-exp over the vocabulary logits
+ *   dlm_refine_update     commit masked positions, edit confident changes,
+ *                         remask the k least confident positions
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Tensors are passed as dlm_tensor descriptors: a DEVICE pointer of the
+ *   current CUDA device, a dtype, the shape and the strides in elements.
+ *   The caller owns every buffer; the library allocates no device memory and
+ *   keeps no pointer after a call returns.
+ * - Calls are asynchronous on the stream set by dlm_set_stream for the calling
+ *   thread (default: the legacy default stream). Outputs are valid once that
+ *   stream has been synchronised. Arguments are validated on the host before
+ *   any launch; a nonzero return means nothing was launched.
+ * - Values that live in device memory (sequence and prompt lengths) cannot be
+ *   checked on the host: the kernels clamp them into range and record
+ *   DLM_DEVERR_LENGTH in the device error word (dlm_get_device_error).
+ * - Return value: DLM_OK (0) or a negative dlm_status. dlm_last_error() gives
+ *   a message for the most recent failure on the calling thread.
+ */
+#ifndef DLMREFINE_H_
+#define DLMREFINE_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DLM_VERSION_MAJOR 0
+#define DLM_VERSION_MINOR 1
+#define DLM_VERSION_PATCH 0
+
+typedef enum dlm_dtype {
+  DLM_BF16 = 1, /* bfloat16 */
+  DLM_F32 = 2,  /* IEEE binary32 */
+  DLM_I32 = 3,  /* int32 */
+  DLM_U8 = 4    /* uint8 */
+} dlm_dtype;
+
+typedef enum dlm_status {
+  DLM_OK = 0,
+  DLM_ERR_NULL = -1,        /* a required pointer or descriptor is NULL */
+  DLM_ERR_DTYPE = -2,       /* unsupported or mismatched dtype */
+  DLM_ERR_SHAPE = -3,       /* rank or extents inconsistent */
+  DLM_ERR_STRIDE = -4,      /* innermost dimension not contiguous, or an unsupported stride */
+  DLM_ERR_ALIGN = -5,       /* base pointer or stride not aligned as required */
+  DLM_ERR_ARG = -6,         /* a scalar argument out of range (NaN threshold, ...) */
+  DLM_ERR_CUDA = -7,        /* a CUDA runtime call or launch failed */
+  DLM_ERR_DEVICE = -8,      /* the device error word was set (dlm_get_device_error) */
+  DLM_ERR_UNSUPPORTED = -9  /* no kernel for this device or configuration */
+} dlm_status;
+
+/* Bits of the device error word. */
+#define DLM_DEVERR_LENGTH 0x1   /* a seq_len / prompt_len outside [0, L] was clamped */
+#define DLM_DEVERR_TIMEOUT 0x2  /* a bounded wait in a kernel gave up; its outputs are undefined */
+#define DLM_DEVERR_NAN 0x4      /* a NaN confidence reached the remask selection */
+
+typedef struct dlm_tensor {
+  void* data;        /* device pointer; 16-byte aligned where a call requires it */
+  int32_t dtype;     /* dlm_dtype */
+  int32_t ndim;      /* 1..4 */
+  int64_t shape[4];  /* extents, outermost first */
+  int64_t stride[4]; /* strides in ELEMENTS, outermost first; stride[ndim-1] must be 1 */
+} dlm_tensor;
+
+/*
+ * Parameters of the refine update (one pass).
+ *   edit_threshold  tau: a filled response position whose argmax differs from
+ *                   its token is edited iff conf >= tau (fp32 compare). Not NaN.
+ *   remask_k        >= 0: remask min(remask_k, r_b) positions per sequence;
+ *                   < 0: remask floor(remask_frac * r_b) (remask_frac in [0, 1]).
+ *   mask_id         the token written at remasked positions.
+ *   prompt_lens     device int32[B]: p_b, clamped into [0, n_b].
+ *   seq_lens        device int32[B]: n_b, clamped into [0, L].
+ * The response of sequence b is [p_b, n_b) and r_b = n_b - p_b.
+ */
+typedef struct dlm_refine_params {
+  float edit_threshold;
+  int32_t remask_k;
+  float remask_frac;
+  int32_t mask_id;
+  const int32_t* prompt_lens;
+  const int32_t* seq_lens;
+} dlm_refine_params;
+
+/*
+ * Step A1 -- non-causal GQA attention (Sec. 4.2: bidirectional correction
+ * over the entire sequence; no causal or block mask, cf. Sec. 3.3).
+ *
+ *   out[b,i,h,:] = sum_{j<n_b} softmax_j(q[b,i,h,:] . k[b,j,g,:] / sqrt(D)) v[b,j,g,:]
+ *   with g = floor(h * Hkv / Hq), for i < n_b; out[b,i,h,:] = 0 for i >= n_b.
+ *
+ *   q, out    [B, L, Hq, D]    BF16 or F32 (both the same dtype)
+ *   k, v      [B, L, Hkv, D]   same dtype as q; Hq % Hkv == 0
+ *   seq_lens  [B] I32          n_b; NULL means n_b = L for all b
+ *   D in {64, 128}. Strides are free except that the innermost dimension is
+ *   contiguous. BF16: tensor cores (tcgen05) with fp32 accumulation and
+ *   softmax, every base pointer and every stride a multiple of 16 bytes.
+ *   F32: fp32 throughout on the CUDA cores.
+ * Key/value rows j >= n_b are never read into a result (they may hold any
+ * bit pattern). out must not overlap q, k or v.
+ */
+int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v,
+                   const dlm_tensor* seq_lens, dlm_tensor* out);
+
+/*
+ * Step A2 -- per-position reduction over the vocabulary (the confidences the
+ * refine threshold of Table 10 and the confident edits of Appendix C.4 act on).
+ *
+ *   m         = max_v logits[r, v]
+ *   argmax[r] = lowest v with logits[r, v] == m
+ *   lse[r]    = m + ln sum_v exp(logits[r, v] - m)
+ *   conf[r]   = exp(m - lse[r])          (the maximum softmax probability)
+ *
+ *   logits  [N, V] or [B, L, V]   BF16 or F32; innermost contiguous; rows may
+ *                                 be strided (row stride in elements)
+ *   argmax  N I32, conf N F32, lse N F32 (any rank with N elements, contiguous)
+ * Math in fp32 with an fp32-accurate exp2; the argmax compare is exact.
+ * Entries may be -inf; a NaN entry or a row of only -inf gives undefined
+ * results for that row. V >= 1.
+ */
+int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf,
+                         dlm_tensor* lse);
+
+/*
+ * Step A3 -- the refine update (prompt fixed, any response position revisable,
+ * Sec. 4.2; token editing with confident edits, Appendix C.4 / Table 11).
+ * For each sequence b, independently:
+ *   1. prompt [0,p_b) and padding [n_b,L) are copied unchanged;
+ *   2. response position i becomes unmasked and takes argmax[i] if it was
+ *      masked (commit), argmax[i] if argmax[i] != tokens[i] and
+ *      conf[i] >= edit_threshold (edit, counted), else tokens[i];
+ *   3. k_b = remask_k >= 0 ? min(remask_k, r_b) : floor(remask_frac * r_b);
+ *   4. the k_b response positions first in (conf ascending, index ascending)
+ *      order are remasked: new_mask = 1, new_tokens = mask_id (-0.0 == +0.0);
+ *   5. n_edits[b] = number of edits of step 2 (commits excluded; an edit that
+ *      step 4 remasks still counts).
+ *
+ *   tokens, new_tokens  [B, L] I32      mask, new_mask  [B, L] U8
+ *   argmax              [B, L] I32      conf            [B, L] F32
+ *   n_edits             [B]    I32
+ * Results are bit-exact: integer work and exact fp32 comparisons only.
+ * new_tokens / new_mask may alias tokens / mask exactly (in-place update);
+ * no other overlap is allowed. L <= 2^24.
+ */
+int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
+                      const dlm_tensor* conf, const dlm_refine_params* params,
+                      dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits);
+
+/* Sets the CUDA stream (a cudaStream_t) used by later calls on this thread. */
+int dlm_set_stream(void* stream);
+/* The stream currently set for this thread. */
+void* dlm_get_stream(void);
+
+/* Static description of a status code. */
+const char* dlm_status_string(int status);
+/* Message for the most recent failure on this thread ("" if none). */
+const char* dlm_last_error(void);
+/* MAJOR * 10000 + MINOR * 100 + PATCH. */
+int dlm_version(void);
+
+/*
+ * Reads the device error word of the current device into *bits (DLM_DEVERR_*),
+ * clearing it if clear != 0. Synchronises the current device. Returns DLM_OK,
+ * or DLM_ERR_CUDA if the device could not be read.
+ */
+int dlm_get_device_error(int32_t* bits, int clear);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DLMREFINE_H_ */

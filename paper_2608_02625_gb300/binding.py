@@ -1,0 +1,164 @@
+"""Thin Python binding of libdlmrefine (argument marshalling only).
+
+Each function has the name and argument order of its C entry point
+(include/dlmrefine.h), takes torch CUDA tensors, builds the dlm_tensor
+descriptors, sets the library's stream to torch's current stream of the
+tensors' device and calls the library. All computation runs in the CUDA
+kernels; a nonzero status raises DlmError. The shared library must have been
+built (``python -m paper_2608_02625_gb300.build``): there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+library_path = os.path.join(_PKG, "libdlmrefine.so")
+
+DLM_BF16, DLM_F32, DLM_I32, DLM_U8 = 1, 2, 3, 4
+_DTYPES = {torch.bfloat16: DLM_BF16, torch.float32: DLM_F32, torch.int32: DLM_I32, torch.uint8: DLM_U8}
+
+
+class DlmTensor(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("dtype", ctypes.c_int32), ("ndim", ctypes.c_int32),
+                ("shape", ctypes.c_int64 * 4), ("stride", ctypes.c_int64 * 4)]
+
+
+class DlmRefineParams(ctypes.Structure):
+    _fields_ = [("edit_threshold", ctypes.c_float), ("remask_k", ctypes.c_int32),
+                ("remask_frac", ctypes.c_float), ("mask_id", ctypes.c_int32),
+                ("prompt_lens", ctypes.c_void_p), ("seq_lens", ctypes.c_void_p)]
+
+
+class DlmError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"libdlmrefine status {status}: {message}")
+        self.status = status
+
+
+def _load():
+    if not os.path.exists(library_path):
+        raise ImportError(f"{library_path} is missing: build it with "
+                          "`python -m paper_2608_02625_gb300.build` (no CPU fallback exists)")
+    lib = ctypes.CDLL(library_path)
+    P = ctypes.POINTER(DlmTensor)
+    lib.dlm_bidir_attn.argtypes = [P, P, P, P, P]
+    lib.dlm_vocab_confidence.argtypes = [P, P, P, P]
+    lib.dlm_refine_update.argtypes = [P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
+    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_set_stream",
+              "dlm_version", "dlm_get_device_error"):
+        getattr(lib, f).restype = ctypes.c_int
+    lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
+    lib.dlm_get_stream.restype = ctypes.c_void_p
+    lib.dlm_status_string.restype = ctypes.c_char_p
+    lib.dlm_status_string.argtypes = [ctypes.c_int]
+    lib.dlm_last_error.restype = ctypes.c_char_p
+    lib.dlm_get_device_error.argtypes = [ctypes.POINTER(ctypes.c_int32), ctypes.c_int]
+    return lib
+
+
+lib = _load()
+
+
+def describe(t: torch.Tensor | None) -> DlmTensor | None:
+    """dlm_tensor descriptor of a tensor (no copy)."""
+    if t is None:
+        return None
+    if t.dtype not in _DTYPES:
+        raise TypeError(f"unsupported dtype {t.dtype}")
+    if t.dim() < 1 or t.dim() > 4:
+        raise ValueError("tensors of rank 1..4 only")
+    d = DlmTensor()
+    d.data = t.data_ptr() if t.numel() else None
+    d.dtype = _DTYPES[t.dtype]
+    d.ndim = t.dim()
+    for i in range(t.dim()):
+        d.shape[i] = t.shape[i]
+        d.stride[i] = t.stride(i)
+    return d
+
+
+def _ref(d):
+    return ctypes.byref(d) if d is not None else None
+
+
+def _check(status: int):
+    if status != 0:
+        msg = lib.dlm_last_error().decode() or lib.dlm_status_string(status).decode()
+        raise DlmError(status, msg)
+
+
+def _prepare(*tensors):
+    dev = None
+    for t in tensors:
+        if t is None:
+            continue
+        if not t.is_cuda:
+            raise ValueError("libdlmrefine takes CUDA tensors")
+        if dev is None:
+            dev = t.device
+        elif t.device != dev:
+            raise ValueError("all tensors must be on one device")
+    torch.cuda.set_device(dev)
+    _check(lib.dlm_set_stream(ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)))
+
+
+def dlm_version() -> int:
+    return lib.dlm_version()
+
+
+def dlm_status_string(status: int) -> str:
+    return lib.dlm_status_string(status).decode()
+
+
+def dlm_bidir_attn(q, k, v, seq_lens, out):
+    """Non-causal GQA attention: out[b,i,h] = softmax(q k^T / sqrt(D)) v over keys j < n_b."""
+    _prepare(q, k, v, seq_lens, out)
+    dq, dk, dv, ds, do = (describe(t) for t in (q, k, v, seq_lens, out))
+    _check(lib.dlm_bidir_attn(_ref(dq), _ref(dk), _ref(dv), _ref(ds), _ref(do)))
+    return out
+
+
+def dlm_vocab_confidence(logits, argmax, conf, lse):
+    """Per row: argmax (lowest index), max softmax probability, log-sum-exp."""
+    _prepare(logits, argmax, conf, lse)
+    ds = [describe(t) for t in (logits, argmax, conf, lse)]
+    _check(lib.dlm_vocab_confidence(*[_ref(d) for d in ds]))
+    return argmax, conf, lse
+
+
+@dataclasses.dataclass
+class RefineParams:
+    edit_threshold: float
+    remask_k: int
+    remask_frac: float
+    mask_id: int
+    prompt_lens: torch.Tensor  # int32 [B] on the device
+    seq_lens: torch.Tensor     # int32 [B] on the device
+
+    def to_c(self) -> DlmRefineParams:
+        for t in (self.prompt_lens, self.seq_lens):
+            if t.dtype != torch.int32 or not t.is_cuda or not t.is_contiguous():
+                raise ValueError("prompt_lens / seq_lens must be contiguous int32 CUDA tensors")
+        return DlmRefineParams(float(self.edit_threshold), int(self.remask_k), float(self.remask_frac),
+                               int(self.mask_id), self.prompt_lens.data_ptr(), self.seq_lens.data_ptr())
+
+
+def dlm_refine_update(tokens, mask, argmax, conf, params: RefineParams, new_tokens, new_mask, n_edits):
+    """Commit masked positions, edit confident changes, remask the k least confident."""
+    _prepare(tokens, mask, argmax, conf, new_tokens, new_mask, n_edits, params.prompt_lens, params.seq_lens)
+    ds = [describe(t) for t in (tokens, mask, argmax, conf)]
+    outs = [describe(t) for t in (new_tokens, new_mask, n_edits)]
+    cp = params.to_c()
+    _check(lib.dlm_refine_update(*[_ref(d) for d in ds], ctypes.byref(cp), *[_ref(d) for d in outs]))
+    return new_tokens, new_mask, n_edits
+
+
+def device_error(clear: bool = True) -> int:
+    """The device error word (DLM_DEVERR_* bits) of the current device; synchronises."""
+    bits = ctypes.c_int32(0)
+    _check(lib.dlm_get_device_error(ctypes.byref(bits), 1 if clear else 0))
+    return bits.value

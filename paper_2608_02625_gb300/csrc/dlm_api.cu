@@ -1,0 +1,340 @@
+// libdlmrefine C ABI: argument validation, stream and error state, dispatch.
+//
+// Every entry point validates its descriptors on the host and returns a
+// negative dlm_status before any launch when something is wrong. Values that
+// live in device memory (lengths) are clamped by the kernels, which record it
+// in the per-device error word read by dlm_get_device_error.
+#include <cstdarg>
+#include <cmath>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "dlm_internal.h"
+#include "dlmrefine.h"
+
+namespace {
+
+// The device error word. Kernels receive its device address (taken once per
+// device with cudaGetSymbolAddress) as an argument.
+__device__ int g_dlm_device_error;
+
+thread_local cudaStream_t t_stream = nullptr;
+thread_local char t_last_error[512] = "";
+
+constexpr int kMaxDevices = 64;
+std::mutex g_err_mu;
+int* g_err_addr[kMaxDevices] = {};
+
+int64_t elem_size(int dtype) {
+  switch (dtype) {
+    case DLM_BF16: return 2;
+    case DLM_F32: return 4;
+    case DLM_I32: return 4;
+    case DLM_U8: return 1;
+    default: return 0;
+  }
+}
+
+int64_t numel(const dlm_tensor* t) {
+  int64_t n = 1;
+  for (int i = 0; i < t->ndim; ++i) n *= t->shape[i];
+  return n;
+}
+
+// Checks pointer, dtype, rank, non-negative extents and a contiguous innermost
+// dimension. `name` appears in the error message.
+int check_tensor(const dlm_tensor* t, const char* name, int dtype_mask, int ndim_lo, int ndim_hi) {
+  using dlm::fail;
+  if (!t) return fail(DLM_ERR_NULL, "%s: descriptor is NULL", name);
+  if (elem_size(t->dtype) == 0 || !((1 << t->dtype) & dtype_mask))
+    return fail(DLM_ERR_DTYPE, "%s: unsupported dtype %d", name, t->dtype);
+  if (t->ndim < ndim_lo || t->ndim > ndim_hi)
+    return fail(DLM_ERR_SHAPE, "%s: rank %d not in [%d, %d]", name, t->ndim, ndim_lo, ndim_hi);
+  for (int i = 0; i < t->ndim; ++i) {
+    if (t->shape[i] < 0) return fail(DLM_ERR_SHAPE, "%s: negative extent", name);
+    if (t->shape[i] > 0x7FFFFFFFLL) return fail(DLM_ERR_SHAPE, "%s: extent too large", name);
+  }
+  if (numel(t) > 0) {
+    if (!t->data) return fail(DLM_ERR_NULL, "%s: data pointer is NULL", name);
+    if (t->shape[t->ndim - 1] > 1 && t->stride[t->ndim - 1] != 1)
+      return fail(DLM_ERR_STRIDE, "%s: innermost dimension must be contiguous", name);
+    for (int i = 0; i < t->ndim; ++i)
+      if (t->stride[i] < 0) return fail(DLM_ERR_STRIDE, "%s: negative stride", name);
+    if (reinterpret_cast<uintptr_t>(t->data) % static_cast<uintptr_t>(elem_size(t->dtype)) != 0)
+      return fail(DLM_ERR_ALIGN, "%s: data pointer not aligned to its element size", name);
+  }
+  return DLM_OK;
+}
+
+bool is_dense(const dlm_tensor* t) {
+  int64_t expect = 1;
+  for (int i = t->ndim - 1; i >= 0; --i) {
+    if (t->shape[i] > 1 && t->stride[i] != expect) return false;
+    expect *= t->shape[i];
+  }
+  return true;
+}
+
+// Byte range [lo, hi) touched by a strided tensor.
+void byte_span(const dlm_tensor* t, uintptr_t* lo, uintptr_t* hi) {
+  int64_t last = 0;
+  for (int i = 0; i < t->ndim; ++i)
+    if (t->shape[i] > 0) last += (t->shape[i] - 1) * t->stride[i];
+  *lo = reinterpret_cast<uintptr_t>(t->data);
+  *hi = *lo + static_cast<uintptr_t>((last + 1) * elem_size(t->dtype));
+}
+
+bool overlaps(const dlm_tensor* a, const dlm_tensor* b) {
+  if (numel(a) == 0 || numel(b) == 0) return false;
+  uintptr_t alo, ahi, blo, bhi;
+  byte_span(a, &alo, &ahi);
+  byte_span(b, &blo, &bhi);
+  return alo < bhi && blo < ahi;
+}
+
+bool same_view(const dlm_tensor* a, const dlm_tensor* b) {
+  if (a->data != b->data || a->ndim != b->ndim || a->dtype != b->dtype) return false;
+  for (int i = 0; i < a->ndim; ++i)
+    if (a->shape[i] != b->shape[i] || (a->shape[i] > 1 && a->stride[i] != b->stride[i])) return false;
+  return true;
+}
+
+constexpr int kMaskBF16F32 = (1 << DLM_BF16) | (1 << DLM_F32);
+
+}  // namespace
+
+namespace dlm {
+
+int fail(int status, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(t_last_error, sizeof(t_last_error), fmt, ap);
+  va_end(ap);
+  return status;
+}
+
+int* device_error_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_err_mu);
+  if (!g_err_addr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_dlm_device_error) != cudaSuccess) return nullptr;
+    g_err_addr[dev] = static_cast<int*>(ptr);
+  }
+  return g_err_addr[dev];
+}
+
+}  // namespace dlm
+
+extern "C" {
+
+int dlm_version(void) { return DLM_VERSION_MAJOR * 10000 + DLM_VERSION_MINOR * 100 + DLM_VERSION_PATCH; }
+
+const char* dlm_status_string(int status) {
+  switch (status) {
+    case DLM_OK: return "ok";
+    case DLM_ERR_NULL: return "null pointer";
+    case DLM_ERR_DTYPE: return "unsupported or mismatched dtype";
+    case DLM_ERR_SHAPE: return "inconsistent shape";
+    case DLM_ERR_STRIDE: return "unsupported stride";
+    case DLM_ERR_ALIGN: return "misaligned pointer or stride";
+    case DLM_ERR_ARG: return "scalar argument out of range";
+    case DLM_ERR_CUDA: return "CUDA error";
+    case DLM_ERR_DEVICE: return "device-side error recorded";
+    case DLM_ERR_UNSUPPORTED: return "unsupported device or configuration";
+    default: return "unknown status";
+  }
+}
+
+const char* dlm_last_error(void) { return t_last_error; }
+
+int dlm_set_stream(void* stream) {
+  t_stream = static_cast<cudaStream_t>(stream);
+  return DLM_OK;
+}
+
+void* dlm_get_stream(void) { return t_stream; }
+
+int dlm_get_device_error(int32_t* bits, int clear) {
+  if (!bits) return dlm::fail(DLM_ERR_NULL, "dlm_get_device_error: bits is NULL");
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return dlm::fail(DLM_ERR_CUDA, "device synchronize: %s", cudaGetErrorString(e));
+  int v = 0;
+  e = cudaMemcpyFromSymbol(&v, g_dlm_device_error, sizeof(int));
+  if (e != cudaSuccess) return dlm::fail(DLM_ERR_CUDA, "read error word: %s", cudaGetErrorString(e));
+  if (clear) {
+    const int zero = 0;
+    e = cudaMemcpyToSymbol(g_dlm_device_error, &zero, sizeof(int));
+    if (e != cudaSuccess) return dlm::fail(DLM_ERR_CUDA, "clear error word: %s", cudaGetErrorString(e));
+  }
+  *bits = v;
+  return DLM_OK;
+}
+
+int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v, const dlm_tensor* seq_lens,
+                   dlm_tensor* out) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  int st;
+  if ((st = check_tensor(q, "q", kMaskBF16F32, 4, 4))) return st;
+  if ((st = check_tensor(k, "k", kMaskBF16F32, 4, 4))) return st;
+  if ((st = check_tensor(v, "v", kMaskBF16F32, 4, 4))) return st;
+  if ((st = check_tensor(out, "out", kMaskBF16F32, 4, 4))) return st;
+  if (k->dtype != q->dtype || v->dtype != q->dtype || out->dtype != q->dtype)
+    return fail(DLM_ERR_DTYPE, "q, k, v and out must share one dtype");
+  const int64_t B = q->shape[0], L = q->shape[1], Hq = q->shape[2], D = q->shape[3];
+  const int64_t Hkv = k->shape[2];
+  for (int i = 0; i < 4; ++i)
+    if (out->shape[i] != q->shape[i]) return fail(DLM_ERR_SHAPE, "out must have the shape of q");
+  for (int i = 0; i < 4; ++i)
+    if (v->shape[i] != k->shape[i]) return fail(DLM_ERR_SHAPE, "v must have the shape of k");
+  if (k->shape[0] != B || k->shape[1] != L || k->shape[3] != D)
+    return fail(DLM_ERR_SHAPE, "k must be [B, L, Hkv, D] with the B, L, D of q");
+  if (D != 64 && D != 128) return fail(DLM_ERR_SHAPE, "head_dim %lld not supported (64 or 128)", (long long)D);
+  if (B * L > 0 && (Hkv < 1 || Hq < Hkv || Hq % Hkv != 0))
+    return fail(DLM_ERR_SHAPE, "Hq (%lld) must be a positive multiple of Hkv (%lld)", (long long)Hq, (long long)Hkv);
+  if (L > (1 << 24)) return fail(DLM_ERR_SHAPE, "L too large");
+  if (seq_lens) {
+    if ((st = check_tensor(seq_lens, "seq_lens", 1 << DLM_I32, 1, 1))) return st;
+    if (seq_lens->shape[0] != B) return fail(DLM_ERR_SHAPE, "seq_lens must have B entries");
+  }
+  if (overlaps(out, q) || overlaps(out, k) || overlaps(out, v))
+    return fail(DLM_ERR_ARG, "out overlaps an input");
+  if (B == 0 || L == 0 || Hq == 0) return DLM_OK;
+  dlm::AttnArgs a;
+  a.q = q->data;
+  a.k = k->data;
+  a.v = v->data;
+  a.out = out->data;
+  a.seq_lens = seq_lens ? static_cast<const int32_t*>(seq_lens->data) : nullptr;
+  a.B = static_cast<int>(B);
+  a.L = static_cast<int>(L);
+  a.Hq = static_cast<int>(Hq);
+  a.Hkv = static_cast<int>(Hkv);
+  a.D = static_cast<int>(D);
+  for (int i = 0; i < 3; ++i) {
+    a.sq[i] = q->stride[i];
+    a.sk[i] = k->stride[i];
+    a.sv[i] = v->stride[i];
+    a.so[i] = out->stride[i];
+  }
+  if (q->dtype == DLM_BF16) {
+    const dlm_tensor* ts[4] = {q, k, v, out};
+    for (const dlm_tensor* t : ts) {
+      if (reinterpret_cast<uintptr_t>(t->data) % 16 != 0)
+        return fail(DLM_ERR_ALIGN, "bf16 attention needs 16-byte aligned base pointers");
+      for (int i = 0; i < 3; ++i)
+        if ((t->stride[i] * 2) % 16 != 0 || t->stride[i] * 2 >= (1LL << 40))
+          return fail(DLM_ERR_ALIGN, "bf16 attention needs strides that are multiples of 16 bytes");
+    }
+    return dlm::launch_attn_tc_bf16(a, t_stream);
+  }
+  return dlm::launch_attn_f32(a, t_stream);
+}
+
+int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  int st;
+  if ((st = check_tensor(logits, "logits", kMaskBF16F32, 2, 3))) return st;
+  if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 1, 3))) return st;
+  if ((st = check_tensor(conf, "conf", 1 << DLM_F32, 1, 3))) return st;
+  if ((st = check_tensor(lse, "lse", 1 << DLM_F32, 1, 3))) return st;
+  const int nd = logits->ndim;
+  const int64_t V = logits->shape[nd - 1];
+  int64_t N = 1;
+  for (int i = 0; i < nd - 1; ++i) N *= logits->shape[i];
+  int64_t row_stride = logits->stride[nd - 2];
+  if (nd == 3 && logits->shape[1] > 1 && logits->shape[0] > 1 &&
+      logits->stride[0] != logits->shape[1] * logits->stride[1])
+    return fail(DLM_ERR_STRIDE, "logits rows must be evenly strided ([B, L, V] with stride[0] = L * stride[1])");
+  if (N > 0 && V < 1) return fail(DLM_ERR_SHAPE, "V must be >= 1");
+  if (N > 1 && row_stride < V) return fail(DLM_ERR_STRIDE, "logits rows overlap");
+  const dlm_tensor* outs[3] = {argmax, conf, lse};
+  for (const dlm_tensor* t : outs) {
+    if (numel(t) != N) return fail(DLM_ERR_SHAPE, "argmax, conf and lse must have one entry per logits row");
+    if (!is_dense(t)) return fail(DLM_ERR_STRIDE, "argmax, conf and lse must be contiguous");
+    if (overlaps(t, logits)) return fail(DLM_ERR_ARG, "outputs overlap logits");
+  }
+  if (overlaps(argmax, conf) || overlaps(argmax, lse) || overlaps(conf, lse))
+    return fail(DLM_ERR_ARG, "outputs overlap each other");
+  if (N == 0) return DLM_OK;
+  dlm::VocabArgs a;
+  a.logits = logits->data;
+  a.is_bf16 = logits->dtype == DLM_BF16;
+  a.N = N;
+  a.V = V;
+  a.row_stride = N > 1 ? row_stride : V;
+  a.argmax = static_cast<int32_t*>(argmax->data);
+  a.conf = static_cast<float*>(conf->data);
+  a.lse = static_cast<float*>(lse->data);
+  return dlm::launch_vocab_confidence(a, t_stream);
+}
+
+int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
+                      const dlm_tensor* conf, const dlm_refine_params* params, dlm_tensor* new_tokens,
+                      dlm_tensor* new_mask, dlm_tensor* n_edits) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  int st;
+  if ((st = check_tensor(tokens, "tokens", 1 << DLM_I32, 2, 2))) return st;
+  if ((st = check_tensor(mask, "mask", 1 << DLM_U8, 2, 2))) return st;
+  if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 2, 2))) return st;
+  if ((st = check_tensor(conf, "conf", 1 << DLM_F32, 2, 2))) return st;
+  if ((st = check_tensor(new_tokens, "new_tokens", 1 << DLM_I32, 2, 2))) return st;
+  if ((st = check_tensor(new_mask, "new_mask", 1 << DLM_U8, 2, 2))) return st;
+  if ((st = check_tensor(n_edits, "n_edits", 1 << DLM_I32, 1, 1))) return st;
+  if (!params) return fail(DLM_ERR_NULL, "params is NULL");
+  const int64_t B = tokens->shape[0], L = tokens->shape[1];
+  const dlm_tensor* bl[6] = {tokens, mask, argmax, conf, new_tokens, new_mask};
+  for (const dlm_tensor* t : bl)
+    if (t->shape[0] != B || t->shape[1] != L) return fail(DLM_ERR_SHAPE, "all [B, L] tensors must share B and L");
+  if (n_edits->shape[0] != B) return fail(DLM_ERR_SHAPE, "n_edits must have B entries");
+  if (L > (1 << 24)) return fail(DLM_ERR_SHAPE, "L too large (max 2^24)");
+  if (std::isnan(params->edit_threshold)) return fail(DLM_ERR_ARG, "edit_threshold is NaN");
+  if (params->remask_k < 0 && !(params->remask_frac >= 0.f && params->remask_frac <= 1.f))
+    return fail(DLM_ERR_ARG, "remask_frac must be in [0, 1] when remask_k < 0");
+  // Outputs may alias their own input exactly; every other overlap is refused.
+  if (!same_view(new_tokens, tokens) && overlaps(new_tokens, tokens))
+    return fail(DLM_ERR_ARG, "new_tokens partially overlaps tokens");
+  if (!same_view(new_mask, mask) && overlaps(new_mask, mask))
+    return fail(DLM_ERR_ARG, "new_mask partially overlaps mask");
+  const dlm_tensor* ins[4] = {tokens, mask, argmax, conf};
+  const dlm_tensor* outs[3] = {new_tokens, new_mask, n_edits};
+  for (int o = 0; o < 3; ++o)
+    for (int i = 0; i < 4; ++i) {
+      if ((o == 0 && i == 0) || (o == 1 && i == 1)) continue;
+      if (overlaps(outs[o], ins[i])) return fail(DLM_ERR_ARG, "an output overlaps an input");
+    }
+  if (overlaps(new_tokens, new_mask) || overlaps(new_tokens, n_edits) || overlaps(new_mask, n_edits))
+    return fail(DLM_ERR_ARG, "outputs overlap each other");
+  if (B == 0) return DLM_OK;
+  dlm::UpdateArgs a;
+  a.tokens = static_cast<const int32_t*>(tokens->data);
+  a.mask = static_cast<const uint8_t*>(mask->data);
+  a.argmax = static_cast<const int32_t*>(argmax->data);
+  a.conf = static_cast<const float*>(conf->data);
+  a.new_tokens = static_cast<int32_t*>(new_tokens->data);
+  a.new_mask = static_cast<uint8_t*>(new_mask->data);
+  a.n_edits = static_cast<int32_t*>(n_edits->data);
+  a.s_tokens = tokens->stride[0];
+  a.s_mask = mask->stride[0];
+  a.s_argmax = argmax->stride[0];
+  a.s_conf = conf->stride[0];
+  a.s_new_tokens = new_tokens->stride[0];
+  a.s_new_mask = new_mask->stride[0];
+  a.B = static_cast<int>(B);
+  a.L = static_cast<int>(L);
+  a.edit_threshold = params->edit_threshold;
+  a.remask_k = params->remask_k;
+  a.remask_frac = params->remask_frac;
+  a.mask_id = params->mask_id;
+  a.prompt_lens = params->prompt_lens;
+  a.seq_lens = params->seq_lens;
+  return dlm::launch_refine_update(a, t_stream);
+}
+
+}  // extern "C"

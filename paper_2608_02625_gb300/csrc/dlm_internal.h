@@ -1,0 +1,63 @@
+// Host-side interfaces between the C ABI layer (dlm_api.cu) and the kernel
+// launchers. Arguments here are already validated.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "dlmrefine.h"
+
+namespace dlm {
+
+// Device address of the error word of the current device (set up once per device).
+int* device_error_word();
+
+// Records a failure message for dlm_last_error() and returns `status`.
+int fail(int status, const char* fmt, ...);
+
+struct AttnArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  void* out;
+  const int32_t* seq_lens;  // may be null: n_b = L
+  int B, L, Hq, Hkv, D;
+  // strides in elements, (b, l, h) order; the innermost stride is 1
+  int64_t sq[3], sk[3], sv[3], so[3];
+};
+
+int launch_attn_tc_bf16(const AttnArgs& a, cudaStream_t stream);  // tcgen05 path
+int launch_attn_f32(const AttnArgs& a, cudaStream_t stream);      // fp32 CUDA-core path
+
+struct VocabArgs {
+  const void* logits;
+  int is_bf16;
+  int64_t N, V, row_stride;  // row stride in elements
+  int32_t* argmax;
+  float* conf;
+  float* lse;
+};
+
+int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream);
+
+struct UpdateArgs {
+  const int32_t* tokens;
+  const uint8_t* mask;
+  const int32_t* argmax;
+  const float* conf;
+  int32_t* new_tokens;
+  uint8_t* new_mask;
+  int32_t* n_edits;
+  int64_t s_tokens, s_mask, s_argmax, s_conf, s_new_tokens, s_new_mask;  // sequence strides
+  int B, L;
+  float edit_threshold;
+  int32_t remask_k;
+  float remask_frac;
+  int32_t mask_id;
+  const int32_t* prompt_lens;
+  const int32_t* seq_lens;
+};
+
+int launch_refine_update(const UpdateArgs& a, cudaStream_t stream);
+
+}  // namespace dlm

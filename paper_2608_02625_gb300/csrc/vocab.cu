@@ -1,0 +1,299 @@
+// Step A2 -- per-position reduction over the vocabulary logits.
+//
+// For each row x of V logits (the confidences that edits are thresholded on:
+// Table 10's refine threshold, Appendix C.4's confident edits):
+//   m = max x,  argmax = lowest index attaining m,
+//   S = sum exp(x - m),  lse = m + ln S,  conf = 1 / S  (= exp(m - lse)).
+//
+// An HBM-bound stream: every logit is read exactly once with 16-byte
+// non-allocating loads, coalesced across the block. Each thread keeps an
+// online (max, first index, scaled sum) triple; the sum is rescaled only when a
+// 16-byte vector raises the running maximum. Threads combine by warp shuffles,
+// warps through shared memory, and -- when there are too few rows to fill the
+// GPU -- the CTAs of a thread-block cluster that split one row combine through
+// distributed shared memory. No global scratch memory.
+#include <cooperative_groups.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "dlm_common.cuh"
+#include "dlm_internal.h"
+
+namespace cg = cooperative_groups;
+
+namespace dlm {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 4;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct Partial {
+  float m;    // running maximum (exact logit value)
+  int idx;    // lowest index attaining m
+  float s;    // sum of exp(x - m)
+};
+
+// Combines two partials; the lower index wins ties of the maximum.
+__device__ __forceinline__ Partial combine(Partial a, Partial b) {
+  Partial r;
+  r.m = fmaxf(a.m, b.m);
+  if (a.m > b.m) r.idx = a.idx;
+  else if (b.m > a.m) r.idx = b.idx;
+  else r.idx = min(a.idx, b.idx);
+  if (r.m == -INFINITY) {
+    r.s = 0.f;
+  } else {
+    float sa = a.m == -INFINITY ? 0.f : a.s * ex2_approx((a.m - r.m) * kLog2e);
+    float sb = b.m == -INFINITY ? 0.f : b.s * ex2_approx((b.m - r.m) * kLog2e);
+    r.s = sa + sb;
+  }
+  return r;
+}
+
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// Elements of one 16-byte vector as fp32.
+template <bool BF16>
+struct Vec;
+
+template <>
+struct Vec<true> {
+  static constexpr int kN = 8;
+  __device__ __forceinline__ static void unpack(uint4 v, float (&x)[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      x[2 * j] = __uint_as_float(w[j] << 16);
+      x[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+    }
+  }
+  __device__ __forceinline__ static float load1(const void* base, int64_t i) {
+    uint16_t h = static_cast<const uint16_t*>(base)[i];
+    return __uint_as_float(static_cast<uint32_t>(h) << 16);
+  }
+};
+
+template <>
+struct Vec<false> {
+  static constexpr int kN = 4;
+  __device__ __forceinline__ static void unpack(uint4 v, float (&x)[4]) {
+    x[0] = __uint_as_float(v.x);
+    x[1] = __uint_as_float(v.y);
+    x[2] = __uint_as_float(v.z);
+    x[3] = __uint_as_float(v.w);
+  }
+  __device__ __forceinline__ static float load1(const void* base, int64_t i) {
+    return static_cast<const float*>(base)[i];
+  }
+};
+
+// Folds one vector of kN values starting at element index e0 into p.
+template <int kN>
+__device__ __forceinline__ void fold(Partial& p, float& mL, const float (&x)[kN], int e0) {
+  float vm = x[0];
+#pragma unroll
+  for (int j = 1; j < kN; ++j) vm = fmaxf(vm, x[j]);
+  if (vm > p.m) {
+    int first = kN - 1;
+#pragma unroll
+    for (int j = kN - 1; j >= 0; --j)
+      if (x[j] == vm) first = j;
+    p.s = (p.m == -INFINITY) ? 0.f : p.s * ex2_approx((p.m - vm) * kLog2e);
+    p.m = vm;
+    p.idx = e0 + first;
+    mL = vm * kLog2e;
+  }
+  if (p.m != -INFINITY) {
+    if constexpr (kN == 1) {
+      p.s += ex2_approx(fmaf(x[0], kLog2e, -mL));
+    } else {
+      float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+      for (int j = 0; j < kN; j += 2) {
+        a0 += ex2_approx(fmaf(x[j], kLog2e, -mL));
+        a1 += ex2_approx(fmaf(x[j + 1], kLog2e, -mL));
+      }
+      p.s += a0 + a1;
+    }
+  }
+}
+
+// Reduces the block's partials into thread 0's return value.
+__device__ __forceinline__ Partial block_reduce(Partial p) {
+  __shared__ Partial warp_part[kThreads / 32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    Partial q;
+    q.m = __shfl_xor_sync(0xffffffffu, p.m, o);
+    q.idx = __shfl_xor_sync(0xffffffffu, p.idx, o);
+    q.s = __shfl_xor_sync(0xffffffffu, p.s, o);
+    p = combine(p, q);
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) warp_part[warp] = p;
+  __syncthreads();
+  if (warp == 0) {
+    p = lane < kThreads / 32 ? warp_part[lane] : Partial{-INFINITY, 0x7FFFFFFF, 0.f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      Partial q;
+      q.m = __shfl_xor_sync(0xffffffffu, p.m, o);
+      q.idx = __shfl_xor_sync(0xffffffffu, p.idx, o);
+      q.s = __shfl_xor_sync(0xffffffffu, p.s, o);
+      p = combine(p, q);
+    }
+  }
+  return p;
+}
+
+// Scans elements [e_begin, e_end) of one row.
+template <bool BF16, bool VEC>
+__device__ __forceinline__ Partial scan_range(const char* row, int64_t e_begin, int64_t e_end) {
+  using VT = Vec<BF16>;
+  constexpr int kN = VT::kN;
+  Partial p{-INFINITY, 0x7FFFFFFF, 0.f};
+  float mL = 0.f;
+  if constexpr (VEC) {
+    // e_begin and e_end are multiples of kN except possibly the row's end.
+    const int64_t v_begin = e_begin / kN;
+    const int64_t v_end = e_end / kN;  // full vectors
+    const uint4* vp = reinterpret_cast<const uint4*>(row);
+    int64_t vi = v_begin + threadIdx.x;
+    for (; vi + (kUnroll - 1) * kThreads < v_end; vi += kUnroll * kThreads) {
+      uint4 raw[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) raw[u] = ld_stream16(vp + vi + u * kThreads);
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        float x[kN];
+        VT::unpack(raw[u], x);
+        fold<kN>(p, mL, x, static_cast<int>((vi + u * kThreads) * kN));
+      }
+    }
+    for (; vi < v_end; vi += kThreads) {
+      float x[kN];
+      VT::unpack(ld_stream16(vp + vi), x);
+      fold<kN>(p, mL, x, static_cast<int>(vi * kN));
+    }
+    e_begin = v_end * kN;  // scalar tail (row length not a multiple of kN)
+  }
+  for (int64_t e = e_begin + threadIdx.x; e < e_end; e += kThreads) {
+    float x[1] = {VT::load1(row, e)};
+    fold<1>(p, mL, x, static_cast<int>(e));
+  }
+  return p;
+}
+
+__device__ __forceinline__ void write_out(const VocabArgs& a, int64_t rowi, Partial p) {
+  a.argmax[rowi] = p.idx;
+  a.conf[rowi] = 1.0f / p.s;
+  a.lse[rowi] = p.m + logf(p.s);
+}
+
+// One CTA per row (grid-stride over rows).
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kThreads, 4) vocab_rows_kernel(VocabArgs a) {
+  const int esz = BF16 ? 2 : 4;
+  for (int64_t rowi = blockIdx.x; rowi < a.N; rowi += gridDim.x) {
+    const char* row = static_cast<const char*>(a.logits) + rowi * a.row_stride * esz;
+    Partial p = scan_range<BF16, VEC>(row, 0, a.V);
+    p = block_reduce(p);
+    if (threadIdx.x == 0) write_out(a, rowi, p);
+    __syncthreads();
+  }
+}
+
+// A cluster of `csize` CTAs per row; CTA c scans a contiguous chunk, rank 0
+// combines the chunk partials through distributed shared memory.
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kThreads, 4) vocab_cluster_kernel(VocabArgs a) {
+  __shared__ Partial cta_part;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int csize = static_cast<int>(cluster.num_blocks());
+  const int crank = static_cast<int>(cluster.block_rank());
+  const int esz = BF16 ? 2 : 4;
+  const int kN = BF16 ? 8 : 4;
+  const int64_t rowi = blockIdx.x / csize;
+  const char* row = static_cast<const char*>(a.logits) + rowi * a.row_stride * esz;
+  // Chunk boundaries on whole vectors.
+  const int64_t nvec = (a.V + kN - 1) / kN;
+  const int64_t per = (nvec + csize - 1) / csize;
+  int64_t e0 = crank * per * kN;
+  int64_t e1 = (crank + 1) * per * kN;
+  if (e0 > a.V) e0 = a.V;
+  if (e1 > a.V) e1 = a.V;
+  Partial p = scan_range<BF16, VEC>(row, e0, e1);
+  p = block_reduce(p);
+  if (threadIdx.x == 0) cta_part = p;
+  cluster.sync();
+  if (crank == 0 && threadIdx.x < 32) {
+    Partial q{-INFINITY, 0x7FFFFFFF, 0.f};
+    if (static_cast<int>(threadIdx.x) < csize) q = *cluster.map_shared_rank(&cta_part, threadIdx.x);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      Partial t;
+      t.m = __shfl_xor_sync(0xffffffffu, q.m, o);
+      t.idx = __shfl_xor_sync(0xffffffffu, q.idx, o);
+      t.s = __shfl_xor_sync(0xffffffffu, q.s, o);
+      q = combine(q, t);
+    }
+    if (threadIdx.x == 0) write_out(a, rowi, q);
+  }
+  cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
+}
+
+template <bool BF16, bool VEC>
+int launch_typed(const VocabArgs& a, cudaStream_t stream) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int esz = BF16 ? 2 : 4;
+  const int64_t row_bytes = a.V * esz;
+  const int64_t want_ctas = 4LL * sms;  // resident CTAs at 4 per SM
+  int csize = 1;
+  if (row_bytes >= 65536) {
+    while (csize < 8 && a.N * csize < 2 * want_ctas) csize *= 2;
+  }
+  if (csize == 1) {
+    int64_t grid = a.N < 64LL * want_ctas ? a.N : 64LL * want_ctas;
+    vocab_rows_kernel<BF16, VEC><<<static_cast<unsigned>(grid), kThreads, 0, stream>>>(a);
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(a.N * csize));
+    cfg.blockDim = dim3(kThreads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = csize;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, vocab_cluster_kernel<BF16, VEC>, a);
+    if (e != cudaSuccess)
+      return fail(DLM_ERR_CUDA, "vocab_confidence cluster launch: %s", cudaGetErrorString(e));
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "vocab_confidence launch: %s", cudaGetErrorString(e));
+  return DLM_OK;
+}
+
+}  // namespace
+
+int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream) {
+  if (a.N == 0) return DLM_OK;
+  const int esz = a.is_bf16 ? 2 : 4;
+  const bool vec = (reinterpret_cast<uintptr_t>(a.logits) % 16 == 0) && ((a.row_stride * esz) % 16 == 0);
+  if (a.is_bf16) return vec ? launch_typed<true, true>(a, stream) : launch_typed<true, false>(a, stream);
+  return vec ? launch_typed<false, true>(a, stream) : launch_typed<false, false>(a, stream);
+}
+
+}  // namespace dlm

@@ -1,0 +1,182 @@
+"""The C ABI without a GPU: the libraries load, export every function that
+include/*.h declares, and reject bad arguments on the host before any launch."""
+import ctypes
+import math
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+PKG = os.path.join(ROOT, "paper_2608_02625_gb300")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2608_02625_gb300 import build
+    build.build()
+
+
+def declared_functions(header):
+    text = open(os.path.join(ROOT, "include", header)).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\*\s]+?\b(dlm_\w+)\s*\(", text, flags=re.M)))
+
+
+@pytest.mark.parametrize("header,lib", [("dlmrefine.h", "libdlmrefine.so"), ("dlmsynth.h", "libdlmsynth.so")])
+def test_exports_every_declared_symbol(header, lib):
+    names = declared_functions(header)
+    assert len(names) >= 2
+    so = ctypes.CDLL(os.path.join(PKG, lib))
+    for n in names:
+        assert hasattr(so, n), f"{lib} does not export {n}"
+
+
+def test_version_and_status_strings():
+    from paper_2608_02625_gb300 import binding as B
+    assert B.dlm_version() == 100
+    assert B.dlm_status_string(0) == "ok"
+    assert "dtype" in B.dlm_status_string(-2)
+
+
+# ---- host-side validation: fake device pointers are never dereferenced
+
+def T(dtype, shape, ptr=0x100000, strides=None):
+    from paper_2608_02625_gb300.binding import DlmTensor
+    d = DlmTensor()
+    d.data = ptr
+    d.dtype = dtype
+    d.ndim = len(shape)
+    if strides is None:
+        strides, acc = [], 1
+        for s in reversed(shape):
+            strides.insert(0, acc)
+            acc *= s
+    for i, (s, st) in enumerate(zip(shape, strides)):
+        d.shape[i] = s
+        d.stride[i] = st
+    return d
+
+
+BF16, F32, I32, U8 = 1, 2, 3, 4
+MB = 1 << 26
+
+
+def attn(q, k, v, sl, o):
+    from paper_2608_02625_gb300.binding import lib
+    r = lambda d: ctypes.byref(d) if d is not None else None
+    return lib.dlm_bidir_attn(r(q), r(k), r(v), r(sl), r(o))
+
+
+def good_attn(D=128, dtype=BF16, Hq=8, Hkv=2):
+    return (T(dtype, [2, 16, Hq, D], 1 * MB), T(dtype, [2, 16, Hkv, D], 2 * MB), T(dtype, [2, 16, Hkv, D], 3 * MB),
+            T(I32, [2], 4 * MB), T(dtype, [2, 16, Hq, D], 5 * MB))
+
+
+@pytest.mark.parametrize("case,status", [
+    ("null_q", -1), ("dtype_mismatch", -2), ("int_dtype", -2), ("head_dim_96", -3), ("gqa_not_multiple", -3),
+    ("out_shape", -3), ("seq_lens_shape", -3), ("inner_stride", -4), ("misaligned_bf16", -5),
+    ("out_overlaps_q", -6), ("rank3", -3),
+])
+def test_attn_rejects(case, status):
+    q, k, v, sl, o = good_attn()
+    if case == "null_q":
+        q = None
+    elif case == "dtype_mismatch":
+        k = T(F32, [2, 16, 2, 128], 2 * MB)
+    elif case == "int_dtype":
+        q, k, v, sl, o = good_attn(dtype=I32)
+    elif case == "head_dim_96":
+        q, k, v, sl, o = good_attn(D=96)
+    elif case == "gqa_not_multiple":
+        q, k, v, sl, o = good_attn(Hq=6, Hkv=4)
+    elif case == "out_shape":
+        o = T(BF16, [2, 16, 4, 128], 5 * MB)
+    elif case == "seq_lens_shape":
+        sl = T(I32, [3], 4 * MB)
+    elif case == "inner_stride":
+        q = T(BF16, [2, 16, 8, 128], 1 * MB, strides=[16 * 8 * 256, 8 * 256, 256, 2])
+    elif case == "misaligned_bf16":
+        q = T(BF16, [2, 16, 8, 128], 1 * MB + 2)
+    elif case == "out_overlaps_q":
+        o = T(BF16, [2, 16, 8, 128], 1 * MB + 256)
+    elif case == "rank3":
+        q = T(BF16, [2, 16, 1024], 1 * MB)
+    assert attn(q, k, v, sl, o) == status
+
+
+def vocab(lg, am, cf, ls):
+    from paper_2608_02625_gb300.binding import lib
+    return lib.dlm_vocab_confidence(*(ctypes.byref(d) if d is not None else None for d in (lg, am, cf, ls)))
+
+
+@pytest.mark.parametrize("case,status", [
+    ("null_conf", -1), ("logits_int", -2), ("argmax_f32", -2), ("count_mismatch", -3), ("strided_out", -4),
+    ("outputs_overlap", -6),
+])
+def test_vocab_rejects(case, status):
+    lg, am, cf, ls = T(BF16, [4, 1000], 1 * MB), T(I32, [4], 2 * MB), T(F32, [4], 3 * MB), T(F32, [4], 4 * MB)
+    if case == "null_conf":
+        cf = None
+    elif case == "logits_int":
+        lg = T(I32, [4, 1000], 1 * MB)
+    elif case == "argmax_f32":
+        am = T(F32, [4], 2 * MB)
+    elif case == "count_mismatch":
+        cf = T(F32, [5], 3 * MB)
+    elif case == "strided_out":
+        ls = T(F32, [4], 4 * MB, strides=[2])
+    elif case == "outputs_overlap":
+        ls = T(F32, [4], 3 * MB + 4)
+    assert vocab(lg, am, cf, ls) == status
+
+
+def update(params, **over):
+    from paper_2608_02625_gb300.binding import lib
+    d = dict(tok=T(I32, [2, 8], 1 * MB), msk=T(U8, [2, 8], 2 * MB), am=T(I32, [2, 8], 3 * MB),
+             cf=T(F32, [2, 8], 4 * MB), nt=T(I32, [2, 8], 5 * MB), nm=T(U8, [2, 8], 6 * MB),
+             ne=T(I32, [2], 7 * MB))
+    d.update(over)
+    r = lambda x: ctypes.byref(x) if x is not None else None
+    return lib.dlm_refine_update(r(d["tok"]), r(d["msk"]), r(d["am"]), r(d["cf"]),
+                                 ctypes.byref(params) if params is not None else None,
+                                 r(d["nt"]), r(d["nm"]), r(d["ne"]))
+
+
+def P(**kw):
+    from paper_2608_02625_gb300.binding import DlmRefineParams
+    base = dict(edit_threshold=0.8, remask_k=2, remask_frac=0.0, mask_id=99, prompt_lens=8 * MB, seq_lens=9 * MB)
+    base.update(kw)
+    return DlmRefineParams(**base)
+
+
+@pytest.mark.parametrize("case,status", [
+    ("null_params", -1), ("nan_threshold", -6), ("frac_above_one", -6), ("frac_nan", -6), ("mask_dtype", -2),
+    ("shape_mismatch", -3), ("n_edits_shape", -3), ("partial_alias", -6), ("output_overlaps_input", -6),
+])
+def test_update_rejects(case, status):
+    if case == "null_params":
+        assert update(None) == status
+    elif case == "nan_threshold":
+        assert update(P(edit_threshold=math.nan)) == status
+    elif case == "frac_above_one":
+        assert update(P(remask_k=-1, remask_frac=1.5)) == status
+    elif case == "frac_nan":
+        assert update(P(remask_k=-1, remask_frac=math.nan)) == status
+    elif case == "mask_dtype":
+        assert update(P(), msk=T(I32, [2, 8], 2 * MB)) == status
+    elif case == "shape_mismatch":
+        assert update(P(), am=T(I32, [2, 9], 3 * MB)) == status
+    elif case == "n_edits_shape":
+        assert update(P(), ne=T(I32, [3], 7 * MB)) == status
+    elif case == "partial_alias":
+        assert update(P(), nt=T(I32, [2, 8], 1 * MB + 4)) == status
+    elif case == "output_overlaps_input":
+        assert update(P(), nt=T(I32, [2, 8], 4 * MB)) == status
+
+
+def test_last_error_message():
+    from paper_2608_02625_gb300.binding import lib
+    q, k, v, sl, o = good_attn(D=96)
+    assert attn(q, k, v, sl, o) == -3
+    assert b"head_dim" in lib.dlm_last_error()

@@ -1,0 +1,145 @@
+"""Step A1 (non-causal GQA attention) on the GPU against the oracle.
+
+bf16: max abs error <= 2e-2 on paper-shaped inputs (q, k, v ~ N(0,1)/sqrt(128));
+peaked inputs (sigma >= 1) use 2e-2 + 1e-2 |ref| (see gpu_util). fp32: 1e-5.
+Output rows i >= n_b must be exactly zero."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import ATTN_RTOL_PEAKED, ATTN_TOL_BF16, ATTN_TOL_F32, dev, host_qkv_seq
+from paper_2608_02625_gb300 import synth, workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_attn(q, k, v, seq_lens, out=None):
+    from paper_2608_02625_gb300 import binding as Bn
+    if out is None:
+        out = torch.full(q.shape, float("nan"), dtype=q.dtype, device=q.device)
+    sl = torch.tensor(np.asarray(seq_lens, dtype=np.int32), device=q.device) if seq_lens is not None else None
+    Bn.dlm_bidir_attn(q, k, v, sl, out)
+    torch.cuda.synchronize()
+    assert Bn.device_error(clear=True) == 0
+    return out
+
+
+def compare(out_gpu: torch.Tensor, ref: np.ndarray, seq_lens, tol_abs, tol_rel=0.0, where=""):
+    g = out_gpu.float().cpu().numpy()
+    B = g.shape[0]
+    for b in range(B):
+        n = int(seq_lens[b]) if seq_lens is not None else g.shape[1]
+        assert np.all(g[b, n:] == 0.0), f"{where}: padded rows of sequence {b} are not zero"
+    err = np.abs(g - ref)
+    bound = tol_abs + tol_rel * np.abs(ref)
+    worst = np.unravel_index(np.argmax(err - bound), err.shape)
+    assert np.all(np.isfinite(g)), f"{where}: non-finite output"
+    assert np.all(err <= bound), (f"{where}: max abs err {err.max():.3g} at {worst} "
+                                  f"(gpu {g[worst]:.5g} ref {ref[worst]:.5g})")
+    return float(err.max()), float(err.max() / max(np.abs(ref).max(), 1e-30))
+
+
+def rand_qkv(B, L, Hq, Hkv, D, sigma, dtype, seed):
+    g = torch.Generator().manual_seed(seed)
+    dt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    q = (torch.randn(B, L, Hq, D, generator=g) * sigma).to(dt)
+    k = (torch.randn(B, L, Hkv, D, generator=g) * sigma).to(dt)
+    v = torch.randn(B, L, Hkv, D, generator=g).to(dt)
+    return q, k, v
+
+
+def run_case(B, L, Hq, Hkv, D, seq_lens, sigma, dtype="bf16", seed=0):
+    q, k, v = rand_qkv(B, L, Hq, Hkv, D, sigma, dtype, seed)
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(),
+                            seq_lens if seq_lens is not None else [L] * B)
+    out = gpu_attn(q.to(dev()), k.to(dev()), v.to(dev()), seq_lens)
+    if dtype == "f32":
+        return compare(out, ref, seq_lens, ATTN_TOL_F32)
+    peaked = sigma >= 0.5
+    return compare(out, ref, seq_lens, ATTN_TOL_BF16, ATTN_RTOL_PEAKED if peaked else 0.0)
+
+
+@pytest.mark.parametrize("sigma", [1 / math.sqrt(128), 1.0, 2.0])
+@pytest.mark.parametrize("B,L,Hq,Hkv,D,sl", [
+    (2, 300, 8, 2, 128, [300, 130]),          # several tiles + ragged tail, varlen
+    (1, 128, 4, 4, 128, [128]),               # MHA: tiles paired across row blocks
+    (2, 384, 6, 2, 128, [384, 257]),          # odd group size: pairs cross heads and rows
+    (1, 50, 2, 1, 128, [50]),                 # L below one tile
+    (3, 256, 4, 2, 64, [256, 1, 129]),        # head_dim 64
+    (6, 260, 2, 1, 128, [0, 1, 127, 128, 129, 260]),  # edge lengths
+])
+def test_bf16_cases(B, L, Hq, Hkv, D, sl, sigma):
+    run_case(B, L, Hq, Hkv, D, sl, sigma, "bf16", seed=B * L + Hq)
+
+
+@pytest.mark.parametrize("B,L,Hq,Hkv,D,sl", [(1, 128, 4, 2, 64, [128]), (2, 200, 4, 1, 128, [200, 77])])
+def test_f32_cases(B, L, Hq, Hkv, D, sl):
+    run_case(B, L, Hq, Hkv, D, sl, 1.0, "f32", seed=3)
+
+
+def test_padding_garbage_never_read():
+    """Key/value rows >= n_b full of NaN/Inf must not reach any output."""
+    B, L, Hq, Hkv, D = 2, 256, 4, 2, 128
+    q, k, v = rand_qkv(B, L, Hq, Hkv, D, 1.0, "bf16", 21)
+    sl = [200, 131]
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(), sl)
+    for b, n in enumerate(sl):
+        k[b, n:] = float("inf")
+        v[b, n:] = float("nan")
+        q[b, n:] = float("nan")
+    out = gpu_attn(q.to(dev()), k.to(dev()), v.to(dev()), sl)
+    compare(out, ref, sl, ATTN_TOL_BF16, ATTN_RTOL_PEAKED, "garbage padding")
+
+
+def test_strided_views_of_packed_qkv():
+    B, L, Hq, Hkv, D = 2, 256, 8, 2, 128
+    packed = (torch.randn(B, L, Hq + 2 * Hkv, D) * 0.5).to(torch.bfloat16)
+    q, k, v = packed[:, :, :Hq], packed[:, :, Hq:Hq + Hkv], packed[:, :, Hq + Hkv:]
+    sl = [256, 100]
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(), sl)
+    pd = packed.to(dev())
+    out = gpu_attn(pd[:, :, :Hq], pd[:, :, Hq:Hq + Hkv], pd[:, :, Hq + Hkv:], sl)
+    compare(out, ref, sl, ATTN_TOL_BF16, ATTN_RTOL_PEAKED, "packed qkv")
+
+
+def test_no_seq_lens_means_full_length():
+    B, L, Hq, Hkv, D = 1, 200, 2, 1, 128
+    q, k, v = rand_qkv(B, L, Hq, Hkv, D, 1.0, "bf16", 5)
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(), [L])
+    out = gpu_attn(q.to(dev()), k.to(dev()), v.to(dev()), None)
+    compare(out, ref, None, ATTN_TOL_BF16, ATTN_RTOL_PEAKED, "no seq_lens")
+
+
+@pytest.mark.parametrize("name,pairs", [
+    ("c1_tiny_f32", "all"),
+    ("c2_single_512", "all"),
+    ("c3_batch32_512", [(0, 0), (5, 13), (17, 31), (31, 7)]),
+    ("c4_long_2048", [(0, 0), (3, 17), (7, 31)]),
+    ("c5_heavy_4step", [(0, 0), (64, 9), (127, 15)]),
+])
+def test_workload_full_size(name, pairs):
+    """The bench's launch (all sequences, all heads); the oracle recomputes the
+    listed (sequence, query head) pairs from host-generated inputs."""
+    from paper_2608_02625_gb300 import synth_gpu
+    w = workloads.get(name)
+    q, k, v = synth_gpu.qkv(w, 0, dev())
+    n = w.seq_lens()
+    out = gpu_attn(q, k, v, n)
+    if pairs == "all":
+        pairs = [(b, h) for b in range(w.B) for h in range(w.Hq)]
+    tol = ATTN_TOL_F32 if w.dtype == "f32" else ATTN_TOL_BF16
+    by_b = {}
+    for b, h in pairs:
+        by_b.setdefault(b, []).append(h)
+    g_out = out.float()
+    for b, heads in by_b.items():
+        hq = host_qkv_seq(w, 0, synth.S_Q, b, w.Hq)
+        hk = host_qkv_seq(w, 0, synth.S_K, b, w.Hkv)
+        hv = host_qkv_seq(w, 0, synth.S_V, b, w.Hkv)
+        for h in heads:
+            g = (h * w.Hkv) // w.Hq
+            ref = oracle.bidir_attn(hq[None, :, h:h + 1], hk[None, :, g:g + 1], hv[None, :, g:g + 1], [n[b]])
+            compare(g_out[b:b + 1, :, h:h + 1], ref, [n[b]], tol, where=f"{name} b={b} h={h}")

@@ -1,0 +1,123 @@
+"""One whole refine step (A1 -> A2 -> A3) and the four-step chain on the GPU.
+
+Update parity follows the decision-margin protocol: GPU and oracle conf may
+differ within tolerance, which can flip a decision only at a position whose
+conf lies within that tolerance of the edit threshold or of the k-th smallest
+response conf. Token, mask and edit count must be identical everywhere else,
+and identical outright when no such position exists."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import ambiguous_positions, check_vocab, dev, host_logit_rows
+from paper_2608_02625_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_step(w, step, q, k, v, logits, tok, msk, prompt, seqlen):
+    from paper_2608_02625_gb300 import binding as Bn
+    d = dev()
+    out = torch.empty_like(q)
+    Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    Bn.dlm_vocab_confidence(logits, am, cf, ls)
+    nt = torch.empty_like(tok)
+    nm = torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    params = Bn.RefineParams(w.edit_threshold[step], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
+    Bn.dlm_refine_update(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), params, nt, nm, ne)
+    torch.cuda.synchronize()
+    assert Bn.device_error(clear=True) == 0
+    return out, am, cf, ls, nt, nm, ne
+
+
+def compare_update(w, step, seqs, state, ref_vocab, gpu_upd, where):
+    """Oracle update of sequences `seqs` (on the oracle's conf) against the GPU's."""
+    tok, msk = state
+    am_ref, cf_ref, _ = ref_vocab
+    p, n = w.prompt_lens()[seqs], w.seq_lens()[seqs]
+    ref = oracle.refine_update(tok, msk, am_ref, cf_ref, edit_threshold=w.edit_threshold[step],
+                               remask_k=w.remask_k, remask_frac=w.remask_frac, mask_id=w.mask_id,
+                               prompt_lens=p, seq_lens=n)
+    g_tok, g_msk, g_ne = gpu_upd
+    amb = ambiguous_positions(w, step, cf_ref, state, am_ref, p, n)
+    diff = (g_tok != ref[0]) | (g_msk != ref[1])
+    assert not np.any(diff & ~amb), f"{where}: update differs at unambiguous positions {np.argwhere(diff & ~amb)[:8]}"
+    for i in range(len(seqs)):
+        if not amb[i].any():
+            assert g_ne[i] == ref[2][i], f"{where}: n_edits of sequence {seqs[i]}"
+    return ref, int(amb.sum()), int(diff.sum())
+
+
+@pytest.mark.parametrize("name,seqs", [("c1_tiny_f32", [0]), ("c2_single_512", [0]), ("c3_batch32_512", [0, 19]),
+                                       ("c4_long_2048", [5])])
+def test_single_step(name, seqs):
+    from paper_2608_02625_gb300 import synth_gpu
+    w = workloads.get(name)
+    d = dev()
+    tok, msk = w.initial_state()
+    q, k, v = synth_gpu.qkv(w, 0, d)
+    logits = synth_gpu.logits(w, 0, d)
+    prompt = torch.from_numpy(w.prompt_lens()).to(d)
+    seqlen = torch.from_numpy(w.seq_lens()).to(d)
+    _, am, cf, ls, nt, nm, ne = gpu_step(w, 0, q, k, v, logits, torch.from_numpy(tok).to(d),
+                                         torch.from_numpy(msk).to(d), prompt, seqlen)
+    rows = np.concatenate([np.arange(b * w.L, (b + 1) * w.L) for b in seqs])
+    ref_vocab = oracle.vocab_confidence(host_logit_rows(w, 0, rows))
+    check_vocab(am.cpu().numpy()[rows], cf.cpu().numpy()[rows], ls.cpu().numpy()[rows], *ref_vocab, where=name)
+    shp = (len(seqs), w.L)
+    ref_v = tuple(a.reshape(shp) for a in ref_vocab)
+    g = (nt.cpu().numpy()[seqs], nm.cpu().numpy()[seqs], ne.cpu().numpy()[seqs])
+    compare_update(w, 0, seqs, (tok[seqs], msk[seqs]), ref_v, g, name)
+
+
+def test_four_step_chain():
+    """c5: 128 x 640, four steps whose logits plant peaks on the current tokens.
+    The GPU runs the whole batch; the oracle runs sequences 0 and 1 (the
+    generator makes them identical to a batch of two) through its own chain."""
+    from paper_2608_02625_gb300 import synth_gpu
+    w = workloads.get("c5_heavy_4step")
+    d = dev()
+    seqs = [0, 1]
+    tok, msk = w.initial_state()
+    g_tok, g_msk = torch.from_numpy(tok).to(d), torch.from_numpy(msk).to(d)
+    o_tok, o_msk = tok[seqs].copy(), msk[seqs].copy()
+    prompt = torch.from_numpy(w.prompt_lens()).to(d)
+    seqlen = torch.from_numpy(w.seq_lens()).to(d)
+    p, n = w.prompt_lens(), w.seq_lens()
+    logits = torch.empty((w.N, w.V), dtype=torch.bfloat16, device=d)
+    diverged = False
+    for s in range(w.steps):
+        q, k, v = synth_gpu.qkv(w, s, d)
+        synth_gpu.logits(w, s, d, g_tok, g_msk, out=logits)
+        prev_tok, prev_msk = g_tok.cpu().numpy(), g_msk.cpu().numpy()
+        _, am, cf, ls, nt, nm, ne = gpu_step(w, s, q, k, v, logits, g_tok, g_msk, prompt, seqlen)
+        a_tok, a_msk, a_ne = nt.cpu().numpy(), nm.cpu().numpy(), ne.cpu().numpy()
+        am_np = am.cpu().numpy().reshape(w.B, w.L)
+        # properties that hold at any size, on every sequence
+        for b in range(w.B):
+            assert np.array_equal(a_tok[b, :p[b]], prev_tok[b, :p[b]])
+            assert int(a_msk[b, p[b]:n[b]].sum()) == min(w.remask_k, n[b] - p[b])
+            keep = (a_msk[b, p[b]:n[b]] == 0)
+            ok = (a_tok[b, p[b]:n[b]] == am_np[b, p[b]:n[b]]) | (a_tok[b, p[b]:n[b]] == prev_tok[b, p[b]:n[b]])
+            assert np.all(ok[keep])
+            assert 0 <= a_ne[b] <= n[b] - p[b]
+        # oracle chain on sequences 0 and 1
+        if not diverged:
+            rows = np.concatenate([np.arange(b * w.L, (b + 1) * w.L) for b in seqs])
+            x = host_logit_rows(w, s, rows, o_tok.reshape(-1), o_msk.reshape(-1))
+            ref_vocab = oracle.vocab_confidence(x)
+            shp = (len(seqs), w.L)
+            ref_v = tuple(a.reshape(shp) for a in ref_vocab)
+            if np.array_equal(prev_tok[seqs], o_tok):
+                check_vocab(am.cpu().numpy()[rows], cf.cpu().numpy()[rows], ls.cpu().numpy()[rows], *ref_vocab,
+                            where=f"step {s}")
+            ref, n_amb, n_diff = compare_update(w, s, seqs, (o_tok, o_msk), ref_v,
+                                                (a_tok[seqs], a_msk[seqs], a_ne[seqs]), f"step {s}")
+            o_tok, o_msk = ref[0], ref[1]
+            diverged = n_diff > 0   # a tolerated flip at an ambiguous position: chains part ways
+        g_tok, g_msk = nt, nm

@@ -1,0 +1,105 @@
+"""Step A2 (vocabulary reduction) on the GPU against the oracle.
+
+argmax is bit-exact (exact compare, lowest index wins); conf and lse are within
+the relative tolerances of gpu_util."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import check_vocab, dev, host_logit_rows
+from paper_2608_02625_gb300 import synth, workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_vocab(x: torch.Tensor):
+    from paper_2608_02625_gb300 import binding as Bn
+    N = x.shape[0] if x.dim() == 2 else x.shape[0] * x.shape[1]
+    am = torch.full((N,), -1, dtype=torch.int32, device=x.device)
+    cf = torch.full((N,), -1.0, dtype=torch.float32, device=x.device)
+    ls = torch.full((N,), -1.0, dtype=torch.float32, device=x.device)
+    Bn.dlm_vocab_confidence(x, am, cf, ls)
+    torch.cuda.synchronize()
+    return am.cpu().numpy(), cf.cpu().numpy(), ls.cpu().numpy()
+
+
+def to_dev(x_f32: np.ndarray, dtype: str) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(x_f32, dtype=np.float32))
+    return (t.to(torch.bfloat16) if dtype == "bf16" else t).to(dev())
+
+
+@pytest.mark.parametrize("name", ["c1_tiny_f32", "c2_single_512"])
+def test_workload_all_rows(name):
+    w = workloads.get(name)
+    from paper_2608_02625_gb300 import synth_gpu
+    x = synth_gpu.logits(w, 0, dev())
+    am, cf, ls = gpu_vocab(x)
+    rows = np.arange(w.N)
+    ref = oracle.vocab_confidence(host_logit_rows(w, 0, rows))
+    check_vocab(am, cf, ls, *ref, where=name)
+
+
+@pytest.mark.parametrize("name", ["c3_batch32_512", "c4_long_2048", "c5_heavy_4step"])
+def test_workload_sampled_rows(name):
+    """Full-size launch; the oracle recomputes a spread sample of rows one by one."""
+    w = workloads.get(name)
+    from paper_2608_02625_gb300 import synth_gpu
+    tok, msk = w.initial_state()
+    t_tok = torch.from_numpy(tok.reshape(-1)).to(dev())
+    t_msk = torch.from_numpy(msk.reshape(-1)).to(dev())
+    x = synth_gpu.logits(w, 0, dev(), t_tok, t_msk)
+    am, cf, ls = gpu_vocab(x)
+    rng = np.random.default_rng(5)
+    rows = np.unique(np.concatenate([[0, w.N - 1], rng.integers(0, w.N, 40)]))
+    ref = oracle.vocab_confidence(host_logit_rows(w, 0, rows, tok.reshape(-1)[rows], msk.reshape(-1)[rows]))
+    check_vocab(am[rows], cf[rows], ls[rows], *ref, where=name)
+    del x
+    torch.cuda.empty_cache()
+
+
+def planted(N, V, seed, sigma=3.0):
+    rng = np.random.default_rng(seed)
+    return (rng.standard_normal((N, V)) * sigma).astype(np.float32)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("N,V", [(1, 1), (3, 7), (2, 8), (5, 1001), (64, 4096), (1, 151552), (7, 151553),
+                                 (300, 32000)])
+def test_shapes(dtype, N, V):
+    x = planted(N, V, N * 7 + V)
+    t = to_dev(x, dtype)
+    ref = oracle.vocab_confidence(t.float().cpu().numpy())
+    check_vocab(*gpu_vocab(t), *ref, where=f"{dtype} {N}x{V}")
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_ties_and_neg_inf(dtype):
+    N, V = 6, 151552
+    x = planted(N, V, 3)
+    x[0, [5, 77777, 150000]] = 40.0          # ties in different threads / cluster chunks
+    x[1, :] = -np.inf
+    x[1, [123456, 99]] = [2.0, 2.0]          # only two finite entries, tied
+    x[2, ::3] = -np.inf
+    x[3, :] = 1.5                            # all equal
+    x[4, V - 1] = 50.0                       # maximum at the last index
+    x[5, 0] = 50.0
+    t = to_dev(x, dtype)
+    am, cf, ls = gpu_vocab(t)
+    ref = oracle.vocab_confidence(t.float().cpu().numpy())
+    check_vocab(am, cf, ls, *ref, where="ties")
+    assert am[0] == 5 and am[1] == 99 and am[3] == 0 and am[4] == V - 1 and am[5] == 0
+
+
+def test_strided_rows_and_3d():
+    N, V = 40, 5000
+    wide = to_dev(planted(N, V + 24, 11), "bf16")
+    x = wide[:, 8:8 + V]                     # rows 16-byte aligned, row stride V + 24
+    ref = oracle.vocab_confidence(x.float().cpu().numpy())
+    check_vocab(*gpu_vocab(x), *ref, where="strided")
+    x3 = to_dev(planted(4 * 10, V, 12), "bf16").reshape(4, 10, V)
+    ref3 = oracle.vocab_confidence(x3.reshape(40, V).float().cpu().numpy())
+    check_vocab(*gpu_vocab(x3), *ref3, where="3d")
+    odd = wide[:, 3:3 + V]                   # rows not 16-byte aligned: scalar path
+    ref_odd = oracle.vocab_confidence(odd.float().cpu().numpy())
+    check_vocab(*gpu_vocab(odd), *ref_odd, where="unaligned")
