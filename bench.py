@@ -60,7 +60,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -70,7 +70,7 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
 
     def __exit__(self, *exc):
         if self.proc:
@@ -80,10 +80,17 @@ class ClockSampler:
             except Exception:
                 self.proc.kill()
 
-    def summary(self):
+    def summary(self, t0=None, t1=None):
+        """Median SM clock and active throttle reasons of the samples taken in
+        [t0, t1] (host time); all samples if the window caught none."""
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        lines = [ln for ts, ln in self.lines if t0 is None or t0 <= ts <= t1]
+        window = "timed region"
+        if not lines:
+            lines = [ln for _, ln in self.lines]
+            window = "whole run (no sample inside the timed region)"
+        for ln in lines:
             parts = [x.strip() for x in ln.split(",")]
             if len(parts) < 9:
                 continue
@@ -98,7 +105,7 @@ class ClockSampler:
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "window": window}
 
 
 # ---------------------------------------------------------------- traffic record
@@ -280,6 +287,7 @@ def run_ours(args, rank, world):
         if ev:
             ev[3].record(stream)
 
+    clk = ClockSampler(d.index if d.index is not None else 0).__enter__()
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -292,12 +300,14 @@ def run_ours(args, rank, world):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    with ClockSampler(d.index if d.index is not None else 0) as clk:
-        t_start.record(stream)
-        for i in range(args.steps):
-            step(evs[i])
-        t_end.record(stream)
-        torch.cuda.synchronize()
+    host_t0 = time.time()
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    host_t1 = time.time()
+    clk.__exit__(None, None, None)
     if world > 1:
         dist.barrier()
     total_ms = t_start.elapsed_time(t_end)
@@ -401,7 +411,7 @@ def run_ours(args, rank, world):
     if timer is not None:
         res["cpu_baseline"] = timer.run()
         timer.close()
-    res["clocks"] = clk.summary()
+    res["clocks"] = clk.summary(host_t0, host_t1)
     res["peaks"] = peaks
     return res
 

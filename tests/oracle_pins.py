@@ -241,8 +241,8 @@ def pin_update_golden():
 
 
 def random_update_case(rng, B=6, L=40, V=50, ties=False):
-    p = rng.integers(0, L // 2, B)
-    n = np.minimum(L, p + rng.integers(0, L, B))
+    p = rng.integers(0, L // 2 + 1, B)
+    n = np.minimum(L, p + rng.integers(0, L + 1, B))
     tok = rng.integers(0, V, (B, L)).astype(np.int32)
     m = (rng.random((B, L)) < 0.3).astype(np.uint8)
     tok[m == 1] = V
