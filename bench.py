@@ -247,6 +247,8 @@ def run_ours(args, rank, world):
     from paper_2608_02625_gb300 import synth_gpu, workloads
 
     base = workloads.get(args.config)
+    if args.batch:
+        base = workloads.scaled(base, B=args.batch, name=f"{base.name}_b{args.batch}")
     # Weak scaling: each rank refines its own seeded batch of the same shape.
     w = workloads.scaled(base, seed=base.seed + rank)
     d = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
@@ -254,7 +256,7 @@ def run_ours(args, rank, world):
     peaks = load_peaks()
 
     timer = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.batch:
         timer = OracleTimer(base.name, host_workers())   # spawned before any GPU work
 
     # Inputs resident in HBM.
@@ -444,8 +446,9 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--batch", type=int, default=None, help="override the workload's batch (profiling runs)")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
