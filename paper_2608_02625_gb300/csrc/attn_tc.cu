@@ -6,36 +6,46 @@
 // block-causal pattern it replaces. out = softmax(q k^T / sqrt(D)) v per
 // (sequence, query head), kv head = floor(h * Hkv / Hq), varlen via seq_lens.
 //
-// Work unit: two 128-row query tiles that read the same key/value head of the
-// same sequence (two query heads of one GQA group, or two row blocks of one
-// head), so each 128-key K/V tile that TMA brings into shared memory feeds
-// both. The kernel is persistent: one CTA per SM walks units
-// blockIdx.x, blockIdx.x + gridDim.x, ... and overlaps the next unit's query
-// load and first score MMAs with the current unit's last MMAs and epilogue.
+// Work unit: two 128-row query tiles ("slots") that read the same key/value
+// head of the same sequence (two query heads of one GQA group, or two row
+// blocks of one head), so each key/value tile staged in shared memory feeds
+// both. The kernel is persistent: one CTA per SM walks units blockIdx.x,
+// blockIdx.x + gridDim.x, ...; the next unit's query tiles load as soon as the
+// slot's last score MMA has run, and its first score MMAs overlap the epilogue.
 //
-// Warp roles (320 threads):
-//   warps 0-3  softmax + epilogue of tile slot 0 (thread t owns query row t = TMEM lane t)
-//   warps 4-7  softmax + epilogue of tile slot 1
-//   warp 8     TMA producer (Q per unit and slot; K_0, V_0, K_1, V_1, ... through a
-//              ring of four tile-sized slots, each released as soon as the MMAs
-//              that read it have completed)
-//   warp 9     tensor-memory allocator and MMA issuer (one elected thread)
-// Tensor memory (512 columns x 128 lanes x 32 bit):
-//   S_i = Q_i K_j^T  fp32, columns [128 i, 128 i + 128)
-//   P_i = bf16 softmax numerators, written over the first 64 columns of S_i
-//   O_i = sum_j P_i V_j fp32, columns [256 + D i, 256 + D i + D)
-// MMA order per key tile j: PV_0(j), S_0(j+1), PV_1(j), S_1(j+1); after the
-// last tile of a unit, S_0(0), S_1(0) of the next unit. The tensor pipe
-// executes one thread's tcgen05.mma in issue order, so a score MMA overwrites
-// P_i only after the PV MMA before it has read P_i.
+// Keys are processed in 64-key sub-tiles so that each slot's scores can be
+// double-buffered in tensor memory: the tensor core computes S(j+1) while the
+// softmax warps work on S(j), which keeps the serial chain
+// softmax -> PV -> next scores off the critical path.
+//
+// Warp roles (352 threads):
+//   warps 0-3  softmax + epilogue of slot 0 (thread t owns query row t = TMEM lane t)
+//   warps 4-7  softmax + epilogue of slot 1
+//   warp 8     TMA producer: Q per unit and slot; K_0, K_1, V_0, K_2, V_1, K_3, ...
+//              through a ring of eight sub-tile slots, each released as soon as
+//              the MMAs that read it have completed
+//   warp 9     tensor-memory allocator; MMA issuer of slot 0 (one elected thread)
+//   warp 10    MMA issuer of slot 1
+// Tensor memory (512 columns x 128 lanes x 32 bit), slot i at column 256 i:
+//   S_i buffers 0 and 1   fp32 128 x 64 at +0 and +64 (sub-tile j uses buffer j % 2)
+//   P_i                    bf16 numerators over the first 32 columns of that buffer
+//   O_i = sum_j P_i V_j    fp32 128 x D at +128
+// MMA order of slot i per sub-tile j: PV_i(j), S_i(j+2). The tensor pipe
+// executes one thread's tcgen05.mma in issue order, so S(j+2) overwrites the
+// buffer holding P(j) only after PV(j) has read it. Each slot has its own
+// issuing thread: issue blocks while the tensor pipe's queue is full, so one
+// thread alone would leave the pipe idle during each of its waits.
 // Online softmax in the log2 domain with exp2; the running maximum used for the
-// numerators is raised (and O rescaled) only when it grows by more than 8,
-// which bounds every numerator by 2^8 and leaves the final O / l exact.
+// numerators is raised (and O rescaled, after the previous PV has completed)
+// only when it grows by more than 8, which bounds every numerator by 2^8 and
+// leaves the final O / l exact.
 //
-// Barrier phases: every barrier completes once per event of one stream of
-// events (per slot: query loads, score MMAs, numerator hand-offs, output
-// hand-offs; per ring stage: fills and releases) and each waiter counts the
-// events it has consumed, so parities line up across units without resets.
+// Barrier phases: each barrier completes once per event of one ordered stream
+// (per slot: query loads, score MMAs per buffer, numerator hand-offs, PV
+// completions, output hand-offs; per ring slot: fills and releases) and every
+// waiter counts the events it consumed. Each wait is arranged so that the
+// barrier cannot run two phases ahead of its waiter (the next event needs
+// something the waiter only provides after the wait), so parities never alias.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -49,32 +59,35 @@
 namespace dlm {
 namespace {
 
-constexpr int kTile = 128;          // query rows per tile = keys per K/V tile
-constexpr int kRing = 4;            // K/V ring: 32-KB slots holding K_c, V_c, K_c+1, ...
-constexpr int kThreads = 320;
+constexpr int kTile = 128;          // query rows per tile
+constexpr int kSub = 64;            // keys per sub-tile
+constexpr int kRing = 8;            // K/V ring slots (one sub-tile each)
+constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;
-constexpr int kMmaWarp = 9;
+constexpr int kMmaWarp0 = 9;   // warps 9 and 10 issue the MMAs of slots 0 and 1
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
 struct Smem {
-  static constexpr int kBoxBytes = kTile * 64 * 2;     // one 128 x 64 bf16 TMA box (16 KB)
-  static constexpr int kTileBytes = kTile * D * 2;     // D / 64 boxes
+  static constexpr int kQBoxBytes = kTile * 64 * 2;    // Q box: 128 rows x 64 bf16 (16 KB)
+  static constexpr int kQBytes = kTile * D * 2;        // D / 64 boxes
+  static constexpr int kKvBoxBytes = kSub * 64 * 2;    // K/V box: 64 rows x 64 bf16 (8 KB)
+  static constexpr int kKvBytes = kSub * D * 2;
   static constexpr int kStageBytes = 32 * 32 * 2;      // epilogue staging: 32 rows x 32 bf16
-  alignas(1024) uint8_t q[2][kTileBytes];
-  alignas(1024) uint8_t ring[kRing][kTileBytes];       // K_c, V_c, K_c+1, V_c+1, ...
+  alignas(1024) uint8_t q[2][kQBytes];
+  alignas(1024) uint8_t ring[kRing][kKvBytes];         // K_0, K_1, V_0, K_2, V_1, ...
   alignas(128) uint8_t stage[8][2][kStageBytes];       // per softmax warp, double-buffered
-  uint64_t bar_q[2];          // query tile of slot i landed        (TMA -> MMA)
-  uint64_t bar_qfree[2];      // last score MMA of slot i issued   (MMA -> TMA)
-  uint64_t bar_full[kRing];   // ring slot filled (V padding cleared) (TMA -> MMA)
-  uint64_t bar_empty[kRing];  // ring slot read by its MMAs         (MMA -> TMA)
-  uint64_t bar_s[2];          // S_i ready                          (MMA -> softmax)
-  uint64_t bar_p[2];          // P_i written, O_i rescaled          (softmax -> MMA)
-  uint64_t bar_o[2];          // O_i final for the unit             (MMA -> epilogue)
-  uint64_t bar_ofree[2];      // O_i read out by the epilogue       (epilogue -> MMA)
-  uint64_t bar_vtmp;          // private fill of a partial V tile
-  uint64_t bar_done;          // every MMA of this CTA completed
+  uint64_t bar_q[2];          // query tile of slot i landed          (TMA -> MMA)
+  uint64_t bar_qfree[2];      // last score MMA of slot i completed   (MMA -> TMA)
+  uint64_t bar_full[kRing];   // ring slot filled (V padding cleared)  (TMA -> MMA)
+  uint64_t bar_empty[kRing];  // ring slot read by its MMAs           (MMA -> TMA)
+  uint64_t bar_s[2][2];       // S_i buffer b ready                   (MMA -> softmax)
+  uint64_t bar_p[2][2];       // hand-off n of slot i (P written, O rescaled) on bar_p[i][n % 2] (softmax -> MMA)
+  uint64_t bar_pv[2][2];      // PV number g of slot i completed, on bar_pv[i][g % 2] (MMA -> softmax)
+  uint64_t bar_ofree[2];      // O_i read out by the epilogue         (epilogue -> MMA)
+  uint64_t bar_vtmp;          // private fill of a partial V sub-tile
+  uint64_t bar_done[2];       // every MMA of issuer i completed
   uint32_t tmem_base;
   int abort;
 };
@@ -89,7 +102,7 @@ struct TcParams {
 };
 
 struct Unit {
-  int b, g, n, nkv;
+  int b, g, n, nkv;  // nkv: 64-key sub-tiles
   int head[2], row0[2];
   bool active[2], run[2];
 };
@@ -115,9 +128,13 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
     U.row0[i] = (U.active[i] ? t / p.G : 0) * kTile;
     U.run[i] = U.active[i] && U.row0[i] < n;
   }
-  U.nkv = (U.run[0] || U.run[1]) ? (n + kTile - 1) / kTile : 0;
+  U.nkv = (U.run[0] || U.run[1]) ? (n + kSub - 1) / kSub : 0;
   return U;
 }
+
+// Ring fill order of a unit with nkv sub-tiles: K_0, K_1, then for each j:
+// V_j followed by K_{j+2} (when it exists). The producer and the MMA issuer
+// walk the same order.
 
 // Warp-uniform bounded wait: true only if every lane saw the phase complete.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
@@ -134,8 +151,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   Smem<D>& sm = *reinterpret_cast<Smem<D>*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   constexpr int kBoxes = D / 64;
-  constexpr uint32_t kBoxBytes = Smem<D>::kBoxBytes;
-  constexpr uint32_t kTileBytes = Smem<D>::kTileBytes;
+  constexpr uint32_t kQBoxBytes = Smem<D>::kQBoxBytes;
+  constexpr uint32_t kQBytes = Smem<D>::kQBytes;
+  constexpr uint32_t kKvBoxBytes = Smem<D>::kKvBoxBytes;
+  constexpr uint32_t kKvBytes = Smem<D>::kKvBytes;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -145,22 +164,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.bar_q[i], 1);
       mbar_init(&sm.bar_qfree[i], 1);
-      mbar_init(&sm.bar_s[i], 1);
-      mbar_init(&sm.bar_p[i], 128);
-      mbar_init(&sm.bar_o[i], 1);
+      mbar_init(&sm.bar_s[i][0], 1);
+      mbar_init(&sm.bar_s[i][1], 1);
+      mbar_init(&sm.bar_p[i][0], 128);
+      mbar_init(&sm.bar_p[i][1], 128);
+      mbar_init(&sm.bar_pv[i][0], 1);
+      mbar_init(&sm.bar_pv[i][1], 1);
       mbar_init(&sm.bar_ofree[i], 128);
     }
     for (int r = 0; r < kRing; ++r) {
       mbar_init(&sm.bar_full[r], 1);
-      mbar_init(&sm.bar_empty[r], 1);
+      mbar_init(&sm.bar_empty[r], 2);  // one arrival per MMA issuer
     }
     mbar_init(&sm.bar_vtmp, 1);
-    mbar_init(&sm.bar_done, 1);
+    mbar_init(&sm.bar_done[0], 1);
+    mbar_init(&sm.bar_done[1], 1);
     sm.abort = 0;
     fence_mbar_init();
     fence_proxy_async_smem();
   }
-  if (warp == kMmaWarp) {
+  if (warp == kMmaWarp0) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -172,10 +195,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kProducerWarp) {
     // ================================================================ TMA producer
-    // Ring fills f = 0, 1, 2, ...: K_c at f = 2c, V_c at f = 2c + 1 (c counts the
-    // key tiles of all units of this CTA); slot f % kRing, phase (f / kRing) & 1.
     int q_loads[2] = {0, 0};   // query loads per slot (= bar_q / bar_qfree phases)
-    int fills = 0;             // ring fills issued
+    int fills = 0;             // ring fills issued; slot fills % kRing, phase (fills / kRing) & 1
     int vtmp = 0;              // private partial-V fills
     bool ok = true;
     if (lane == 0) {
@@ -184,8 +205,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tv);
       prefetch_tmap(&to);
     }
-    auto acquire = [&](int f) -> bool {
-      return f < kRing || warp_wait(&sm.bar_empty[f % kRing], ((f / kRing) - 1) & 1, abort, p.err);
+    // Loads K_j (is_v false) or V_j into the next ring slot.
+    auto fill = [&](const Unit& U, int j, bool is_v) -> bool {
+      const int r = fills % kRing;
+      if (fills >= kRing && !warp_wait(&sm.bar_empty[r], ((fills / kRing) - 1) & 1, abort, p.err)) return false;
+      const int valid = U.n - j * kSub;
+      if (!is_v || valid >= kSub) {
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&sm.bar_full[r], kKvBytes);
+          for (int c = 0; c < kBoxes; ++c)
+            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, is_v ? &tv : &tk, &sm.bar_full[r], 64 * c, U.g, j * kSub,
+                        U.b);
+        }
+      } else {
+        // Last, partial value sub-tile: rows >= n may hold any bit pattern and
+        // a zero softmax weight does not cancel a NaN/Inf, so clear them in
+        // shared memory before the MMA reads the tile.
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&sm.bar_vtmp, kKvBytes);
+          for (int c = 0; c < kBoxes; ++c)
+            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, &tv, &sm.bar_vtmp, 64 * c, U.g, j * kSub, U.b);
+        }
+        ++vtmp;
+        if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err)) return false;
+        const int zrows = kSub - valid;
+        for (int c = 0; c < kBoxes; ++c) {
+          uint4* base = reinterpret_cast<uint4*>(sm.ring[r] + c * kKvBoxBytes + valid * 128);
+          for (int e = lane; e < zrows * 8; e += 32) base[e] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.bar_full[r]);
+      }
+      ++fills;
+      return true;
     };
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
       const Unit U = decode_unit(p, unit);
@@ -195,56 +248,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         // The slot's previous query tile is free once its last score MMA has run.
         if (q_loads[i] > 0 && !warp_wait(&sm.bar_qfree[i], (q_loads[i] - 1) & 1, abort, p.err)) { ok = false; break; }
         if (lane == 0) {
-          mbar_arrive_expect_tx(&sm.bar_q[i], kTileBytes);
+          mbar_arrive_expect_tx(&sm.bar_q[i], kQBytes);
           for (int c = 0; c < kBoxes; ++c)
-            tma_load_4d(sm.q[i] + c * kBoxBytes, &tq, &sm.bar_q[i], 64 * c, U.head[i], U.row0[i], U.b);
+            tma_load_4d(sm.q[i] + c * kQBoxBytes, &tq, &sm.bar_q[i], 64 * c, U.head[i], U.row0[i], U.b);
         }
         ++q_loads[i];
       }
+      if (!ok) break;
+      ok = fill(U, 0, false) && (U.nkv < 2 || fill(U, 1, false));
       for (int j = 0; ok && j < U.nkv; ++j) {
-        // K_j
-        if (!acquire(fills)) { ok = false; break; }
-        {
-          const int r = fills % kRing;
-          if (lane == 0) {
-            mbar_arrive_expect_tx(&sm.bar_full[r], kTileBytes);
-            for (int c = 0; c < kBoxes; ++c)
-              tma_load_4d(sm.ring[r] + c * kBoxBytes, &tk, &sm.bar_full[r], 64 * c, U.g, j * kTile, U.b);
-          }
-          ++fills;
-        }
-        // V_j
-        if (!acquire(fills)) { ok = false; break; }
-        const int r = fills % kRing;
-        const int valid = U.n - j * kTile;
-        if (valid >= kTile) {
-          if (lane == 0) {
-            mbar_arrive_expect_tx(&sm.bar_full[r], kTileBytes);
-            for (int c = 0; c < kBoxes; ++c)
-              tma_load_4d(sm.ring[r] + c * kBoxBytes, &tv, &sm.bar_full[r], 64 * c, U.g, j * kTile, U.b);
-          }
-          ++fills;
-        } else {
-          // Last, partial tile: value rows >= n may hold any bit pattern and a
-          // zero softmax weight does not cancel a NaN/Inf, so clear them in
-          // shared memory before the MMA reads the tile.
-          if (lane == 0) {
-            mbar_arrive_expect_tx(&sm.bar_vtmp, kTileBytes);
-            for (int c = 0; c < kBoxes; ++c)
-              tma_load_4d(sm.ring[r] + c * kBoxBytes, &tv, &sm.bar_vtmp, 64 * c, U.g, j * kTile, U.b);
-          }
-          ++vtmp;
-          if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err)) { ok = false; break; }
-          const int zrows = kTile - valid;
-          for (int c = 0; c < kBoxes; ++c) {
-            uint4* base = reinterpret_cast<uint4*>(sm.ring[r] + c * kBoxBytes + valid * 128);
-            for (int e = lane; e < zrows * 8; e += 32) base[e] = make_uint4(0u, 0u, 0u, 0u);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.bar_full[r]);
-          ++fills;
-        }
+        ok = fill(U, j, true) && (j + 2 >= U.nkv || fill(U, j + 2, false));
       }
     }
     // Teardown: let every copy this warp issued land before the block exits.
@@ -258,94 +271,104 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
-    // ================================================================ MMA issuer
+  } else if (warp >= kMmaWarp0) {
+    // ================================================================ MMA issuers
+    // Warp kMmaWarp0 + i issues every MMA of slot i (one elected thread), so the
+    // two slots' MMA streams do not wait on each other's hand-offs; each
+    // stream is ordered on its own. Both issuers arrive on every ring slot's
+    // release barrier: with tcgen05.commit after their MMAs read the slot, or
+    // with a plain arrive (after the fill landed) when their slot idles in a unit.
+    const int i = warp - kMmaWarp0;
     if (lane == 0) {
-      constexpr uint32_t idesc_s = idesc_bf16_f32(128, 128, false, false);  // Q, K both K-major
-      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);     // V is MN-major (D contiguous)
-      const uint32_t q_addr[2] = {smem_u32(sm.q[0]), smem_u32(sm.q[1])};
-      auto issue_s = [&](int i, int r) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(128, kSub, false, false);  // Q, K both K-major
+      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);      // V is MN-major (D contiguous)
+      const uint32_t q_addr = smem_u32(sm.q[i]);
+      const uint32_t s_tmem = tmem + 256 * i;
+      // S_i(j) -> buffer b: Q_i [128 x D] times K sub-tile [64 x D]^T.
+      auto issue_s = [&](int b, int r) {
         const uint32_t kaddr = smem_u32(sm.ring[r]);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
-          mma_ss(tmem + 128 * i, sdesc_sw128(q_addr[i] + off, 16, 1024), sdesc_sw128(kaddr + off, 16, 1024),
+          const uint32_t qoff = (kk / 4) * kQBoxBytes + (kk % 4) * 32;
+          const uint32_t koff = (kk / 4) * kKvBoxBytes + (kk % 4) * 32;
+          mma_ss(s_tmem + kSub * b, sdesc_sw128(q_addr + qoff, 16, 1024), sdesc_sw128(kaddr + koff, 16, 1024),
                  idesc_s, kk > 0);
         }
-        mma_commit(&sm.bar_s[i]);
+        mma_commit(&sm.bar_s[i][b]);
       };
-      auto issue_pv = [&](int i, int r, bool acc) {
+      // O_i (+)= P_i(j) [128 x 64, tensor memory] times V sub-tile [64 x D].
+      int pv_issued = 0;  // PVs issued (all units)
+      auto issue_pv = [&](int b, int r, bool acc) {
         const uint32_t vaddr = smem_u32(sm.ring[r]);
 #pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          mma_ts(tmem + 256 + D * i, tmem + 128 * i + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kBoxBytes, 1024),
+        for (int kk = 0; kk < kSub / 16; ++kk) {
+          mma_ts(s_tmem + 128, s_tmem + kSub * b + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kKvBoxBytes, 1024),
                  idesc_o, (acc || kk > 0) ? 1u : 0u);
         }
+        mma_commit(&sm.bar_pv[i][pv_issued & 1]);
+        ++pv_issued;
       };
       auto wait_fill = [&](int f) -> bool {
         return mbar_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err);
       };
-      int q_loads[2] = {0, 0};   // bar_q phases consumed per slot
-      int units_run[2] = {0, 0}; // bar_o / bar_ofree phases per slot
-      int p_seen[2] = {0, 0};    // bar_p phases consumed per slot
-      int tiles = 0;             // key tiles consumed (ring fill of K_c is 2c, of V_c is 2c + 1)
+      auto release = [&](int f, bool issued) {
+        if (issued) mma_commit(&sm.bar_empty[f % kRing]);
+        else mbar_arrive(&sm.bar_empty[f % kRing]);
+      };
+      int q_loads = 0;    // bar_q phases consumed
+      int units_run = 0;  // bar_ofree phases
+      int p_seen = 0;     // bar_p hand-offs consumed
+      int f = 0;          // ring fills consumed
       bool ok = true;
       for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
         const Unit U = decode_unit(p, unit);
         if (U.nkv == 0) continue;
-        const int last_slot = U.run[1] ? 1 : 0;
-        for (int i = 0; i < 2 && ok; ++i) {
-          if (!U.run[i]) continue;
-          ok = mbar_wait(&sm.bar_q[i], q_loads[i] & 1, abort, p.err);
-          ++q_loads[i];
+        const bool run = U.run[i];
+        if (run) {
+          ok = mbar_wait(&sm.bar_q[i], q_loads & 1, abort, p.err);
+          ++q_loads;
         }
-        if (!ok || !wait_fill(2 * tiles)) break;
-        tc_fence_after();
-        for (int i = 0; i < 2; ++i) {
-          if (!U.run[i]) continue;
-          issue_s(i, (2 * tiles) % kRing);
-          if (U.nkv == 1) mma_commit(&sm.bar_qfree[i]);
+        // Prologue: S(0) and S(1) into buffers 0 and 1.
+        for (int j = 0; ok && j < 2 && j < U.nkv; ++j, ++f) {
+          if (!wait_fill(f)) { ok = false; break; }
+          if (run) {
+            tc_fence_after();
+            issue_s(j, f % kRing);
+            if (j == U.nkv - 1) mma_commit(&sm.bar_qfree[i]);
+          }
+          release(f, run);
         }
-        mma_commit(&sm.bar_empty[(2 * tiles) % kRing]);
         for (int j = 0; ok && j < U.nkv; ++j) {
-          const int c = tiles + j;
-          const int fv = 2 * c + 1, fk = 2 * c + 2;
-          const bool next = j + 1 < U.nkv;
+          const int fv = f++;
           if (!wait_fill(fv)) { ok = false; break; }
-          bool k_ready = false;
-          for (int i = 0; i < 2 && ok; ++i) {
-            if (!U.run[i]) continue;
+          if (run) {
             // O_i of this slot's previous unit must have been read out before PV(0) overwrites it.
-            if (j == 0 && units_run[i] > 0 &&
-                !mbar_wait(&sm.bar_ofree[i], (units_run[i] - 1) & 1, abort, p.err)) {
+            if (j == 0 && units_run > 0 && !mbar_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err)) {
               ok = false;
               break;
             }
-            if (!mbar_wait(&sm.bar_p[i], p_seen[i] & 1, abort, p.err)) { ok = false; break; }
-            ++p_seen[i];
+            if (!mbar_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
+            ++p_seen;
             tc_fence_after();
-            issue_pv(i, fv % kRing, j > 0);
-            if (!next) mma_commit(&sm.bar_o[i]);
-            if (i == last_slot) mma_commit(&sm.bar_empty[fv % kRing]);
-            if (next) {
-              if (!k_ready) {
-                if (!wait_fill(fk)) { ok = false; break; }
-                tc_fence_after();
-                k_ready = true;
-              }
-              issue_s(i, fk % kRing);
-              if (j + 2 == U.nkv) mma_commit(&sm.bar_qfree[i]);
-              if (i == last_slot) mma_commit(&sm.bar_empty[fk % kRing]);
+            issue_pv(j & 1, fv % kRing, j > 0);
+          }
+          release(fv, run);
+          if (j + 2 < U.nkv) {
+            const int fk = f++;
+            if (!wait_fill(fk)) { ok = false; break; }
+            if (run) {
+              tc_fence_after();
+              issue_s(j & 1, fk % kRing);
+              if (j + 2 == U.nkv - 1) mma_commit(&sm.bar_qfree[i]);
             }
+            release(fk, run);
           }
         }
-        tiles += U.nkv;
-        for (int i = 0; i < 2; ++i)
-          if (U.run[i]) ++units_run[i];
+        if (run) ++units_run;
       }
       // Teardown: every MMA issued by this thread completes before TMEM is freed.
-      mma_commit(&sm.bar_done);
-      mbar_drain(&sm.bar_done, 0);
+      mma_commit(&sm.bar_done[i]);
+      mbar_drain(&sm.bar_done[i], 0);
     }
     __syncwarp();
   } else {
@@ -354,11 +377,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int qw = warp & 3;                 // warp within the warpgroup: rows 32 qw .. 32 qw + 31
     const int t = threadIdx.x & 127;         // row within the tile = TMEM lane
     const uint32_t lane_base = static_cast<uint32_t>(qw * 32) << 16;
-    const uint32_t s_addr = tmem + lane_base + 128 * i;
-    const uint32_t o_addr = tmem + lane_base + 256 + D * i;
-    int s_seen = 0;     // bar_s phases consumed
-    int units_run = 0;  // bar_o phases consumed
+    const uint32_t slot_addr = tmem + lane_base + 256 * i;
+    const uint32_t o_addr = slot_addr + 128;
+    int s_seen[2] = {0, 0};  // bar_s phases consumed per buffer
+    // PVs of this slot are numbered g = 0, 1, 2, ... over all units; PV g
+    // completes a phase of bar_pv[i][g % 2]. pv_done = how many have been
+    // consumed (in order), pv_next = number of this slot's sub-tile hand-offs.
+    // At sub-tile hand-off n the softmax has consumed PV n-2 (or n-1); PV n+0
+    // and later need P(n), so neither barrier can run two phases ahead.
+    int pv_done = 0, pv_next = 0;
     bool ok = true;
+    auto consume_pv_upto = [&](int g) -> bool {
+      for (; pv_done <= g; ++pv_done)
+        if (!warp_wait(&sm.bar_pv[i][pv_done & 1], (pv_done >> 1) & 1, abort, p.err)) return false;
+      return true;
+    };
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
       const Unit U = decode_unit(p, unit);
       if (!U.active[i]) continue;
@@ -376,30 +409,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_used = -INFINITY;
       float l = 0.f;
       for (int j = 0; j < U.nkv; ++j) {
-        if (!warp_wait(&sm.bar_s[i], s_seen & 1, abort, p.err)) { ok = false; break; }
-        ++s_seen;
+        const int b = j & 1;
+        const uint32_t s_addr = slot_addr + kSub * b;
+        if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err)) { ok = false; break; }
+        ++s_seen[b];
         tc_fence_after();
-        uint32_t sr[128];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(s_addr + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&sr[32 * c]));
+        uint32_t sr[kSub];
+        tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+        tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
         tmem_wait_ld();
-        float sv[128];
+        float sv[kSub];
 #pragma unroll
-        for (int c = 0; c < 128; ++c) sv[c] = __uint_as_float(sr[c]);
-        const int valid = U.n - j * kTile;
-        if (valid < kTile) {
+        for (int c = 0; c < kSub; ++c) sv[c] = __uint_as_float(sr[c]);
+        const int valid = U.n - j * kSub;
+        if (valid < kSub) {
 #pragma unroll
-          for (int c = 0; c < 128; ++c)
+          for (int c = 0; c < kSub; ++c)
             if (c >= valid) sv[c] = -INFINITY;
         }
         float mx0 = sv[0], mx1 = sv[1], mx2 = sv[2], mx3 = sv[3];
 #pragma unroll
-        for (int c = 4; c < 128; c += 4) {
-          mx0 = fmaxf(mx0, sv[c]);
-          mx1 = fmaxf(mx1, sv[c + 1]);
-          mx2 = fmaxf(mx2, sv[c + 2]);
-          mx3 = fmaxf(mx3, sv[c + 3]);
+        for (int c = 4; c + 8 <= kSub; c += 8) {
+          mx0 = fmax3(mx0, sv[c], sv[c + 1]);
+          mx1 = fmax3(mx1, sv[c + 2], sv[c + 3]);
+          mx2 = fmax3(mx2, sv[c + 4], sv[c + 5]);
+          mx3 = fmax3(mx3, sv[c + 6], sv[c + 7]);
         }
+        mx0 = fmax3(mx0, sv[kSub - 4], sv[kSub - 3]);
+        mx1 = fmax3(mx1, sv[kSub - 2], sv[kSub - 1]);
         const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * p.scale_log2;
         const bool raise = m_tile > m_used + kRescaleThreshold;
         if (__any_sync(0xffffffffu, raise)) {
@@ -408,8 +445,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           l *= alpha;
           m_used = m_new;
           if (j > 0) {
-            // O holds sum_{j' < j} P V (the score MMA of tile j was issued after
-            // the PV MMA of tile j-1, and bar_s has completed): rescale it.
+            // O holds sum_{j' < j} P V once PV(j-1) has completed: rescale it.
+            if (!consume_pv_upto(pv_next - 1)) { ok = false; break; }
+            tc_fence_after();
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
               uint32_t ov[32];
@@ -421,25 +459,36 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        uint32_t pk[64];
-        float l0 = 0.f, l1 = 0.f;
+        // Numerators 2^(s * scale - m), two columns at a time; P goes to tensor
+        // memory (over the first 32 columns of this S buffer) 16 columns at a time.
+        const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
+        const float2 nm2 = make_float2(-m_used, -m_used);
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int c = 0; c < 64; ++c) {
-          const float p0 = ex2_approx(fmaf(sv[2 * c], p.scale_log2, -m_used));
-          const float p1 = ex2_approx(fmaf(sv[2 * c + 1], p.scale_log2, -m_used));
-          l0 += p0;
-          l1 += p1;
-          pk[c] = pack_bf16x2(p0, p1);
+        for (int qq = 0; qq < kSub / 32; ++qq) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const int col = 32 * qq + 2 * c;
+            const float2 x = ffma2(make_float2(sv[col], sv[col + 1]), sc2, nm2);
+            const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+            if (c & 1) acc1 = fadd2(acc1, e); else acc0 = fadd2(acc0, e);
+            pk[c] = pack_bf16x2(e.x, e.y);
+          }
+          tmem_st16(s_addr + 16 * qq, pk);
         }
-        l += l0 + l1;
-        tmem_st32(s_addr, *reinterpret_cast<const uint32_t(*)[32]>(&pk[0]));
-        tmem_st32(s_addr + 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[32]));
+        l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
         tmem_wait_st();
+        // PV two hand-offs back (long complete) is consumed before P(j) goes out.
+        // Hand-off n uses bar_p[i][n % 2]: hand-off n + 2 waits for PV n here,
+        // and PV n is only issued after the MMA thread consumed hand-off n.
+        if (!consume_pv_upto(pv_next - 2)) { ok = false; break; }
         tc_fence_before();
-        mbar_arrive(&sm.bar_p[i]);
+        mbar_arrive(&sm.bar_p[i][pv_next & 1]);
+        ++pv_next;
       }
-      if (!ok || !warp_wait(&sm.bar_o[i], units_run & 1, abort, p.err)) { ok = false; break; }
-      ++units_run;
+      // The unit's last PV.
+      if (!ok || !consume_pv_upto(pv_next - 1)) { ok = false; break; }
       // Epilogue: read O_i out of tensor memory, hand the columns back to the
       // MMA warp, then normalise, convert to bf16, stage 32 rows x 32 columns
       // per warp in shared memory and write them with TMA stores (rows >= n
@@ -490,7 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (warp == kMmaWarp) {
+  if (warp == kMmaWarp0) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -540,8 +589,8 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   CUtensorMap mq, mk, mv, mo;
   int st;
   if ((st = make_map(&mq, a.q, a.B, a.L, a.Hq, D, a.sq)) != DLM_OK) return st;
-  if ((st = make_map(&mk, a.k, a.B, a.L, a.Hkv, D, a.sk)) != DLM_OK) return st;
-  if ((st = make_map(&mv, a.v, a.B, a.L, a.Hkv, D, a.sv)) != DLM_OK) return st;
+  if ((st = make_map(&mk, a.k, a.B, a.L, a.Hkv, D, a.sk, 64, kSub)) != DLM_OK) return st;
+  if ((st = make_map(&mv, a.v, a.B, a.L, a.Hkv, D, a.sv, 64, kSub)) != DLM_OK) return st;
   // Output: 32 x 32 boxes (one warp's rows, one 64-byte column chunk), no swizzle.
   if ((st = make_map(&mo, a.out, a.B, a.L, a.Hq, D, a.so, 32, 32, CU_TENSOR_MAP_SWIZZLE_NONE)) != DLM_OK) return st;
   TcParams p;
