@@ -34,7 +34,10 @@
 // executes one thread's tcgen05.mma in issue order, so S(j+2) overwrites the
 // buffer holding P(j) only after PV(j) has read it. Each slot has its own
 // issuing thread: issue blocks while the tensor pipe's queue is full, so one
-// thread alone would leave the pipe idle during each of its waits.
+// thread alone would leave the pipe idle during each of its waits. At the
+// start of every unit slot 1's softmax waits for slot 0's first hand-off, so
+// the two slots run half a step apart and their MMA bursts alternate with
+// the other slot's softmax instead of coinciding.
 // Online softmax in the log2 domain with exp2; the running maximum used for the
 // numerators is raised (and O rescaled, after the previous PV has completed)
 // only when it grows by more than 8, which bounds every numerator by 2^8 and
@@ -77,7 +80,7 @@ struct Smem {
   static constexpr int kStageBytes = 32 * 32 * 2;      // epilogue staging: 32 rows x 32 bf16
   alignas(1024) uint8_t q[2][kQBytes];
   alignas(1024) uint8_t ring[kRing][kKvBytes];         // K_0, K_1, V_0, K_2, V_1, ...
-  alignas(128) uint8_t stage[8][2][kStageBytes];       // per softmax warp, double-buffered
+  alignas(1024) uint8_t stage[8][2][kStageBytes];       // per softmax warp, double-buffered
   uint64_t bar_q[2];          // query tile of slot i landed          (TMA -> MMA)
   uint64_t bar_qfree[2];      // last score MMA of slot i completed   (MMA -> TMA)
   uint64_t bar_full[kRing];   // ring slot filled (V padding cleared)  (TMA -> MMA)
@@ -90,6 +93,7 @@ struct Smem {
   uint64_t bar_done[2];       // every MMA of issuer i completed
   uint32_t tmem_base;
   int abort;
+  int unit_flag;   // units whose first slot-0 hand-off happened
 };
 
 struct TcParams {
@@ -180,6 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&sm.bar_done[0], 1);
     mbar_init(&sm.bar_done[1], 1);
     sm.abort = 0;
+    sm.unit_flag = 0;
     fence_mbar_init();
     fence_proxy_async_smem();
   }
@@ -380,6 +385,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t slot_addr = tmem + lane_base + 256 * i;
     const uint32_t o_addr = slot_addr + 128;
     int s_seen[2] = {0, 0};  // bar_s phases consumed per buffer
+    int unit_seq = 0;
     // PVs of this slot are numbered g = 0, 1, 2, ... over all units; PV g
     // completes a phase of bar_pv[i][g % 2]. pv_done = how many have been
     // consumed (in order), pv_next = number of this slot's sub-tile hand-offs.
@@ -405,6 +411,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int e = 0; e < D / 8; ++e) dst[e] = make_uint4(0u, 0u, 0u, 0u);
         }
         continue;
+      }
+      ++unit_seq;
+      if (i == 1) {
+        // Start slot 1 one softmax behind slot 0 so that the two slots' MMA
+        // bursts alternate instead of coinciding.
+        uint64_t t0 = global_timer_ns();
+        while (*reinterpret_cast<volatile int*>(&sm.unit_flag) < unit_seq) {
+          if (global_timer_ns() - t0 > kWaitBudgetNs || *abort) { *abort = 1; ok = false; break; }
+        }
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       }
       float m_used = -INFINITY;
       float l = 0.f;
@@ -485,6 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!consume_pv_upto(pv_next - 2)) { ok = false; break; }
         tc_fence_before();
         mbar_arrive(&sm.bar_p[i][pv_next & 1]);
+        if (i == 0 && j == 0 && t == 0) *reinterpret_cast<volatile int*>(&sm.unit_flag) = unit_seq;
         ++pv_next;
       }
       // The unit's last PV.
@@ -492,7 +509,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Epilogue: read O_i out of tensor memory, hand the columns back to the
       // MMA warp, then normalise, convert to bf16, stage 32 rows x 32 columns
       // per warp in shared memory and write them with TMA stores (rows >= n
-      // are zero; rows >= L are clipped by the tensor map).
+      // are zero; rows >= L are clipped by the tensor map). The staging rows
+      // use the 64-byte swizzle of the output tensor map (16-byte chunk e of
+      // row r at position e ^ ((r / 2) % 4)), which makes the warp's stores
+      // free of shared-memory bank conflicts.
       tc_fence_after();
       uint32_t ov[D];
 #pragma unroll
@@ -513,7 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) bulk_wait_read<1>();
             __syncwarp();
           }
-          uint4* dst = reinterpret_cast<uint4*>(buf + lane * 64);
+          uint8_t* dstrow = buf + lane * 64;
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
             uint32_t w[4];
@@ -523,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               w[h] = valid_row ? pack_bf16x2(__uint_as_float(ov[col]) * inv, __uint_as_float(ov[col + 1]) * inv)
                                : 0u;
             }
-            dst[e] = make_uint4(w[0], w[1], w[2], w[3]);
+            *reinterpret_cast<uint4*>(dstrow + ((e ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -592,7 +612,7 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   if ((st = make_map(&mk, a.k, a.B, a.L, a.Hkv, D, a.sk, 64, kSub)) != DLM_OK) return st;
   if ((st = make_map(&mv, a.v, a.B, a.L, a.Hkv, D, a.sv, 64, kSub)) != DLM_OK) return st;
   // Output: 32 x 32 boxes (one warp's rows, one 64-byte column chunk), no swizzle.
-  if ((st = make_map(&mo, a.out, a.B, a.L, a.Hq, D, a.so, 32, 32, CU_TENSOR_MAP_SWIZZLE_NONE)) != DLM_OK) return st;
+  if ((st = make_map(&mo, a.out, a.B, a.L, a.Hq, D, a.so, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)) != DLM_OK) return st;
   TcParams p;
   p.B = a.B;
   p.L = a.L;
