@@ -87,7 +87,8 @@ struct Smem {
   uint64_t bar_empty[kRing];  // ring slot read by its MMAs           (MMA -> TMA)
   uint64_t bar_s[2][2];       // S_i buffer b ready                   (MMA -> softmax)
   uint64_t bar_p[2][2];       // hand-off n of slot i (P written, O rescaled) on bar_p[i][n % 2] (softmax -> MMA)
-  uint64_t bar_pv[2][2];      // PV number g of slot i completed, on bar_pv[i][g % 2] (MMA -> softmax)
+  uint64_t bar_pvm[2];        // the unit's next-to-last PV of slot i completed (MMA -> softmax)
+  uint64_t bar_o[2];          // the unit's last PV of slot i completed: O_i final (MMA -> epilogue)
   uint64_t bar_ofree[2];      // O_i read out by the epilogue         (epilogue -> MMA)
   uint64_t bar_vtmp;          // private fill of a partial V sub-tile
   uint64_t bar_done[2];       // every MMA of issuer i completed
@@ -172,8 +173,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.bar_s[i][1], 1);
       mbar_init(&sm.bar_p[i][0], 128);
       mbar_init(&sm.bar_p[i][1], 128);
-      mbar_init(&sm.bar_pv[i][0], 1);
-      mbar_init(&sm.bar_pv[i][1], 1);
+      mbar_init(&sm.bar_pvm[i], 1);
+      mbar_init(&sm.bar_o[i], 1);
       mbar_init(&sm.bar_ofree[i], 128);
     }
     for (int r = 0; r < kRing; ++r) {
@@ -302,16 +303,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&sm.bar_s[i][b]);
       };
       // O_i (+)= P_i(j) [128 x 64, tensor memory] times V sub-tile [64 x D].
-      int pv_issued = 0;  // PVs issued (all units)
-      auto issue_pv = [&](int b, int r, bool acc) {
+      // Only the unit's last two PVs signal their completion (bar_pvm, bar_o):
+      // for the others, the completion of the score MMA issued after them does.
+      auto issue_pv = [&](int b, int r, bool acc, uint64_t* done) {
         const uint32_t vaddr = smem_u32(sm.ring[r]);
 #pragma unroll
         for (int kk = 0; kk < kSub / 16; ++kk) {
           mma_ts(s_tmem + 128, s_tmem + kSub * b + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kKvBoxBytes, 1024),
                  idesc_o, (acc || kk > 0) ? 1u : 0u);
         }
-        mma_commit(&sm.bar_pv[i][pv_issued & 1]);
-        ++pv_issued;
+        if (done) mma_commit(done);
       };
       auto wait_fill = [&](int f) -> bool {
         return mbar_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err);
@@ -355,7 +356,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
             ++p_seen;
             tc_fence_after();
-            issue_pv(j & 1, fv % kRing, j > 0);
+            issue_pv(j & 1, fv % kRing, j > 0,
+                     j == U.nkv - 1 ? &sm.bar_o[i] : (j == U.nkv - 2 ? &sm.bar_pvm[i] : nullptr));
           }
           release(fv, run);
           if (j + 2 < U.nkv) {
@@ -386,18 +388,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t o_addr = slot_addr + 128;
     int s_seen[2] = {0, 0};  // bar_s phases consumed per buffer
     int unit_seq = 0;
-    // PVs of this slot are numbered g = 0, 1, 2, ... over all units; PV g
-    // completes a phase of bar_pv[i][g % 2]. pv_done = how many have been
-    // consumed (in order), pv_next = number of this slot's sub-tile hand-offs.
-    // At sub-tile hand-off n the softmax has consumed PV n-2 (or n-1); PV n+0
-    // and later need P(n), so neither barrier can run two phases ahead.
-    int pv_done = 0, pv_next = 0;
+    // PV completion: S(j) is issued after PV(j-2) and S(j+1) after PV(j-1)
+    // (one issuer, in order), so waiting for a score buffer also waits for the
+    // PVs before it. Only the unit's last two PVs have barriers of their own
+    // (bar_pvm, bar_o), each consumed once per unit; their next phases need
+    // hand-offs of the next unit, so they cannot run two phases ahead.
+    bool s_ahead[2] = {false, false};  // next phase of bar_s[i][b] already consumed
+    int hand = 0;       // hand-offs so far: hand-off n on bar_p[i][n % 2]
+    int pvm_seen = 0;   // bar_pvm phases consumed
+    int units_run = 0;  // bar_o phases consumed
     bool ok = true;
-    auto consume_pv_upto = [&](int g) -> bool {
-      for (; pv_done <= g; ++pv_done)
-        if (!warp_wait(&sm.bar_pv[i][pv_done & 1], (pv_done >> 1) & 1, abort, p.err)) return false;
-      return true;
-    };
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
       const Unit U = decode_unit(p, unit);
       if (!U.active[i]) continue;
@@ -424,11 +424,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       float m_used = -INFINITY;
       float l = 0.f;
+      bool pvm_done = false;
       for (int j = 0; j < U.nkv; ++j) {
         const int b = j & 1;
         const uint32_t s_addr = slot_addr + kSub * b;
-        if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err)) { ok = false; break; }
-        ++s_seen[b];
+        if (s_ahead[b]) {
+          s_ahead[b] = false;
+        } else {
+          if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err)) { ok = false; break; }
+          ++s_seen[b];
+        }
         tc_fence_after();
         uint32_t sr[kSub];
         tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
@@ -461,8 +466,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           l *= alpha;
           m_used = m_new;
           if (j > 0) {
-            // O holds sum_{j' < j} P V once PV(j-1) has completed: rescale it.
-            if (!consume_pv_upto(pv_next - 1)) { ok = false; break; }
+            // O holds sum_{j' < j} P V once PV(j-1) has completed: wait for the
+            // score MMA issued after it (S(j+1)), or on the unit's last sub-tile
+            // for PV(j-1)'s own barrier, then rescale.
+            if (j + 1 < U.nkv) {
+              const int bn = b ^ 1;
+              if (!warp_wait(&sm.bar_s[i][bn], s_seen[bn] & 1, abort, p.err)) { ok = false; break; }
+              ++s_seen[bn];
+              s_ahead[bn] = true;
+            } else {
+              if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err)) { ok = false; break; }
+              ++pvm_seen;
+              pvm_done = true;
+            }
             tc_fence_after();
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
@@ -495,17 +511,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
         tmem_wait_st();
-        // PV two hand-offs back (long complete) is consumed before P(j) goes out.
-        // Hand-off n uses bar_p[i][n % 2]: hand-off n + 2 waits for PV n here,
-        // and PV n is only issued after the MMA thread consumed hand-off n.
-        if (!consume_pv_upto(pv_next - 2)) { ok = false; break; }
+        // Hand-off n uses bar_p[i][n % 2]; hand-off n + 2 comes after S(n + 2),
+        // which the issuer starts only after consuming hand-off n.
         tc_fence_before();
-        mbar_arrive(&sm.bar_p[i][pv_next & 1]);
+        mbar_arrive(&sm.bar_p[i][hand & 1]);
         if (i == 0 && j == 0 && t == 0) *reinterpret_cast<volatile int*>(&sm.unit_flag) = unit_seq;
-        ++pv_next;
+        ++hand;
       }
-      // The unit's last PV.
-      if (!ok || !consume_pv_upto(pv_next - 1)) { ok = false; break; }
+      // The unit's last two PVs (the next-to-last one only if not consumed above).
+      if (ok && U.nkv >= 2 && !pvm_done) {
+        if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err)) ok = false;
+        ++pvm_seen;
+      }
+      if (!ok || !warp_wait(&sm.bar_o[i], units_run & 1, abort, p.err)) { ok = false; break; }
+      ++units_run;
       // Epilogue: read O_i out of tensor memory, hand the columns back to the
       // MMA warp, then normalise, convert to bf16, stage 32 rows x 32 columns
       // per warp in shared memory and write them with TMA stores (rows >= n

@@ -94,6 +94,24 @@ def test_padding_garbage_never_read():
     compare(out, ref, sl, ATTN_TOL_BF16, ATTN_RTOL_PEAKED, "garbage padding")
 
 
+@pytest.mark.parametrize("L,n", [(300, 300), (256, 250), (128, 128), (200, 129)])
+def test_running_max_rises_every_tile(L, n):
+    """Scores that grow along the keys (k_j = 2 j e_0, q = e_0) raise the
+    running maximum by far more than the rescale threshold in every key
+    sub-tile, the last one included, so the output-rescale path runs each time."""
+    B, Hq, Hkv, D = 1, 4, 2, 128
+    q = torch.zeros(B, L, Hq, D)
+    q[..., 0] = 1.0
+    k = torch.zeros(B, L, Hkv, D)
+    k[0, :, :, 0] = (2.0 * torch.arange(L, dtype=torch.float32))[:, None]
+    g = torch.Generator().manual_seed(9)
+    v = torch.randn(B, L, Hkv, D, generator=g)
+    q, k, v = q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16)
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(), [n])
+    out = gpu_attn(q.to(dev()), k.to(dev()), v.to(dev()), [n])
+    compare(out, ref, [n], ATTN_TOL_BF16, ATTN_RTOL_PEAKED, "rising max")
+
+
 def test_strided_views_of_packed_qkv():
     B, L, Hq, Hkv, D = 2, 256, 8, 2, 128
     packed = (torch.randn(B, L, Hq + 2 * Hkv, D) * 0.5).to(torch.bfloat16)
