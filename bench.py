@@ -236,6 +236,32 @@ def host_workers():
     return max(1, min(16, (os.cpu_count() or 2) - 1))
 
 
+# ---------------------------------------------------------------- multi-GPU (replicas)
+
+def replica_workload(base, rank: int):
+    """Weak scaling: rank r refines its own seeded batch of the base workload's
+    shape; ranks never exchange data."""
+    from paper_2608_02625_gb300 import workloads
+    return workloads.scaled(base, seed=base.seed + rank)
+
+
+def max_over_ranks(value_ms: float, world: int, device) -> float:
+    """The slowest rank's time: the job is done when its last replica is."""
+    if world == 1:
+        return value_ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value_ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_steps_per_s(ms_per_step: float, world: int) -> float:
+    """Whole-job refine steps/s: each of the `world` replicas finishes one
+    step of its own batch every ms_per_step."""
+    return world * 1000.0 / ms_per_step
+
+
 # ---------------------------------------------------------------- GPU arm
 
 def run_ours(args, rank, world):
@@ -250,7 +276,7 @@ def run_ours(args, rank, world):
     if args.batch:
         base = workloads.scaled(base, B=args.batch, name=f"{base.name}_b{args.batch}")
     # Weak scaling: each rank refines its own seeded batch of the same shape.
-    w = workloads.scaled(base, seed=base.seed + rank)
+    w = replica_workload(base, rank)
     d = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(d)
     peaks = load_peaks()
@@ -320,10 +346,7 @@ def run_ours(args, rank, world):
     }
     if Bn.device_error(clear=True):
         raise RuntimeError("device error word set during the timed region")
-    t = torch.tensor([total_ms], dtype=torch.float64, device=d)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, d)
     ms_per_step = total_ms / args.steps
 
     # ---- end to end through the public API with host buffers
@@ -363,11 +386,9 @@ def run_ours(args, rank, world):
             e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
-        te = torch.tensor([e0.elapsed_time(e1) / k_e2e], dtype=torch.float64, device=d)
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * 1000.0 / float(te.item()), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": float(te.item()), "steps": k_e2e}
+        te = max_over_ranks(e0.elapsed_time(e1) / k_e2e, world, d)
+        e2e = {"value": job_steps_per_s(te, world), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": te, "steps": k_e2e}
 
     if rank != 0:
         return None
@@ -395,7 +416,7 @@ def run_ours(args, rank, world):
                 "traffic": recorded_traffic("attn_tc.cu", base.name), "algorithmic_flops": attn_flops,
                 "peak_source": peaks["source"]}
 
-    steps_per_s = world * 1000.0 / ms_per_step
+    steps_per_s = job_steps_per_s(ms_per_step, world)
     res = {
         "metric": METRIC, "value": steps_per_s, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",

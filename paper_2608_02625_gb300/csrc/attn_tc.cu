@@ -249,6 +249,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
       const Unit U = decode_unit(p, unit);
       if (U.nkv == 0) continue;
+      // The unit's first key tiles need only ring slots: start them before
+      // the query tiles, which wait for the previous unit's last score MMAs.
+      ok = fill(U, 0, false) && (U.nkv < 2 || fill(U, 1, false));
       for (int i = 0; i < 2 && ok; ++i) {
         if (!U.run[i]) continue;
         // The slot's previous query tile is free once its last score MMA has run.
@@ -261,7 +264,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++q_loads[i];
       }
       if (!ok) break;
-      ok = fill(U, 0, false) && (U.nkv < 2 || fill(U, 1, false));
       for (int j = 0; ok && j < U.nkv; ++j) {
         ok = fill(U, j, true) && (j + 2 >= U.nkv || fill(U, j + 2, false));
       }
