@@ -112,19 +112,19 @@ class ClockSampler:
 
 def kernel_source_sha(fname: str) -> str:
     h = hashlib.sha256()
-    for f in (fname, "dlm_common.cuh"):
+    for f in (fname, "dlm_common.cuh", "update_impl.cuh"):
         with open(os.path.join(ROOT, "paper_2608_02625_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel_file: str, workload: str):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel source
-    still matches the one profiled (else None)."""
+def recorded_traffic(kernel_file: str, kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    kernel source still matches the one profiled (else None)."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             rec = json.load(f)
-        e = rec[kernel_file][workload]
+        e = rec[kernel_file][kernel][workload]
         if e["source_sha"] != kernel_source_sha(kernel_file):
             return None
         return e["dram_bytes_per_launch"]
@@ -300,7 +300,9 @@ def run_ours(args, rank, world):
     nt, nm = torch.empty_like(tok), torch.empty_like(msk)
     ne = torch.empty(w.B, dtype=torch.int32, device=d)
     params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
+    workspace = torch.zeros(Bn.dlm_refine_step_workspace_bytes(w.B) // 4, dtype=torch.int32, device=d)
     stream = torch.cuda.current_stream(d)
+    fused = args.path == "fused"
 
     def step(ev=None):
         if ev:
@@ -308,6 +310,13 @@ def run_ours(args, rank, world):
         Bn.dlm_bidir_attn(q, k, v, seqlen, out)
         if ev:
             ev[1].record(stream)
+        if fused:
+            Bn.dlm_refine_step(logits, tok, msk, params, am.view(w.B, w.L), cf.view(w.B, w.L), ls.view(w.B, w.L),
+                               nt, nm, ne, workspace)
+            if ev:
+                ev[2].record(stream)
+                ev[3].record(stream)
+            return
         Bn.dlm_vocab_confidence(logits, am, cf, ls)
         if ev:
             ev[2].record(stream)
@@ -404,16 +413,22 @@ def run_ours(args, rank, world):
     }
     kern["attn"]["frac_of_measured_bf16"] = kern["attn"]["achieved_tflops"] / peaks["bf16_tflops"]
     kern["vocab"]["frac_of_measured_hbm"] = kern["vocab"]["achieved_gbs"] / peaks["hbm_gbs"]
+    if fused:   # the vocabulary stream and the update share one launch
+        kern["vocab"]["kernel"] = "vocab_step (vocabulary reduction + update)"
+        kern["update"] = {"ms": 0.0, "fused_into": "vocab"}
     dominant = max(("attn", "vocab"), key=lambda kk: per_kernel[kk])
     if dominant == "vocab":
-        roof = {"kernel": "vocab_confidence", "bound": "hbm", "achieved": kern["vocab"]["achieved_gbs"],
+        roof = {"kernel": "vocab_step" if fused else "vocab_confidence", "bound": "hbm",
+                "achieved": kern["vocab"]["achieved_gbs"],
                 "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": kern["vocab"]["frac_of_measured_hbm"],
-                "traffic": recorded_traffic("vocab.cu", base.name), "algorithmic_bytes": vocab_bytes,
+                "traffic": recorded_traffic("vocab.cu", "vocab_step_kernel" if fused else "vocab_rows_kernel",
+                                            base.name),
+                "algorithmic_bytes": vocab_bytes,
                 "peak_source": peaks["source"]}
     else:
         roof = {"kernel": "bidir_attn", "bound": "tensor", "achieved": kern["attn"]["achieved_tflops"],
                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s", "frac": kern["attn"]["frac_of_measured_bf16"],
-                "traffic": recorded_traffic("attn_tc.cu", base.name), "algorithmic_flops": attn_flops,
+                "traffic": recorded_traffic("attn_tc.cu", "attn_tc_kernel", base.name), "algorithmic_flops": attn_flops,
                 "peak_source": peaks["source"]}
 
     steps_per_s = job_steps_per_s(ms_per_step, world)
@@ -428,7 +443,8 @@ def run_ours(args, rank, world):
         "refined_tokens_per_sec": steps_per_s * w.refined_tokens(),
         "kernels": kern,
         "roofline": roof,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (2 if fused else 3) * args.steps,
+        "path": args.path,
         "e2e": e2e,
     }
     if timer is not None:
@@ -474,6 +490,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="separate", choices=["fused", "separate"],
+                    help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
+                         "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -12,6 +12,8 @@
  *   dlm_refine_update     commit masked positions, edit confident changes,
  *                         remask the k least confident positions
  *
+ * dlm_refine_step does the last two in one launch (same results).
+ *
  * Conventions shared by every call
  * --------------------------------
  * - Tensors are passed as dlm_tensor descriptors: a DEVICE pointer of the
@@ -31,6 +33,7 @@
 #ifndef DLMREFINE_H_
 #define DLMREFINE_H_
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -157,6 +160,37 @@ int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tenso
 int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
                       const dlm_tensor* conf, const dlm_refine_params* params,
                       dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits);
+
+/*
+ * Steps A2 and A3 fused in one launch (the per-position reduction of the
+ * confidences of Table 10 / Appendix C.4 feeding the update of Sec. 4.2).
+ * Computes exactly what dlm_vocab_confidence(logits, argmax, conf, lse)
+ * followed by dlm_refine_update(tokens, mask, argmax, conf, params,
+ * new_tokens, new_mask, n_edits) computes: argmax, conf and lse are written
+ * as by the first call, and the update reads them back. The CTA that finishes
+ * the last row of sequence b runs the update of b, so the update of one
+ * sequence overlaps the vocabulary stream of the others and no second launch
+ * is needed.
+ *
+ *   logits  [B * L, V] or [B, L, V]   BF16 or F32, as for dlm_vocab_confidence
+ *   argmax, conf, lse                 [B, L] contiguous (I32, F32, F32)
+ *   other tensors and params          as for dlm_refine_update
+ *   workspace                         device memory of at least
+ *                                     dlm_refine_step_workspace_bytes(B) bytes,
+ *                                     4-byte aligned, owned by the caller
+ * The workspace holds one row counter per sequence. It must be zero before
+ * its first use (e.g. cudaMemsetAsync); each completed call leaves it zero
+ * again, so it can be reused by later calls without clearing. Calls that
+ * share a workspace must not overlap on the GPU (they would race on the
+ * counters): issue them on one stream. new_tokens / new_mask may alias
+ * tokens / mask exactly; no other overlap among the tensors is allowed.
+ */
+int dlm_refine_step(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* mask,
+                    const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf,
+                    dlm_tensor* lse, dlm_tensor* new_tokens, dlm_tensor* new_mask,
+                    dlm_tensor* n_edits, void* workspace, size_t workspace_bytes);
+/* Bytes of workspace dlm_refine_step needs for a batch of `batch` sequences. */
+size_t dlm_refine_step_workspace_bytes(int64_t batch);
 
 /* Sets the CUDA stream (a cudaStream_t) used by later calls on this thread. */
 int dlm_set_stream(void* stream);

@@ -48,7 +48,11 @@ def _load():
     lib.dlm_bidir_attn.argtypes = [P, P, P, P, P]
     lib.dlm_vocab_confidence.argtypes = [P, P, P, P]
     lib.dlm_refine_update.argtypes = [P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
-    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_set_stream",
+    lib.dlm_refine_step.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P,
+                                    ctypes.c_void_p, ctypes.c_size_t]
+    lib.dlm_refine_step_workspace_bytes.argtypes = [ctypes.c_int64]
+    lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
+    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step", "dlm_set_stream",
               "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
     lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
@@ -155,6 +159,29 @@ def dlm_refine_update(tokens, mask, argmax, conf, params: RefineParams, new_toke
     cp = params.to_c()
     _check(lib.dlm_refine_update(*[_ref(d) for d in ds], ctypes.byref(cp), *[_ref(d) for d in outs]))
     return new_tokens, new_mask, n_edits
+
+
+def dlm_refine_step_workspace_bytes(batch: int) -> int:
+    return lib.dlm_refine_step_workspace_bytes(int(batch))
+
+
+def dlm_refine_step(logits, tokens, mask, params: RefineParams, argmax, conf, lse, new_tokens, new_mask, n_edits,
+                    workspace):
+    """Vocabulary reduction and refine update in one launch.
+
+    workspace: a CUDA tensor of at least dlm_refine_step_workspace_bytes(B) bytes,
+    zero before its first use; each completed call leaves it zero again."""
+    _prepare(logits, tokens, mask, argmax, conf, lse, new_tokens, new_mask, n_edits, workspace,
+             params.prompt_lens, params.seq_lens)
+    if not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
+    ins = [describe(t) for t in (logits, tokens, mask)]
+    outs = [describe(t) for t in (argmax, conf, lse, new_tokens, new_mask, n_edits)]
+    cp = params.to_c()
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(lib.dlm_refine_step(*[_ref(d) for d in ins], ctypes.byref(cp), *[_ref(d) for d in outs],
+                               ctypes.c_void_p(workspace.data_ptr() if nbytes else None), ctypes.c_size_t(nbytes)))
+    return argmax, conf, lse, new_tokens, new_mask, n_edits
 
 
 def device_error(clear: bool = True) -> int:

@@ -28,7 +28,7 @@ LIBS = {
     "libdlmrefine.so": ["dlm_api.cu", "attn_tc.cu", "attn_f32.cu", "vocab.cu", "update.cu"],
     "libdlmsynth.so": ["synth.cu"],
 }
-HEADERS = ["dlm_common.cuh", "dlm_internal.h"]
+HEADERS = ["dlm_common.cuh", "dlm_internal.h", "update_impl.cuh"]
 
 
 def nvcc() -> str:

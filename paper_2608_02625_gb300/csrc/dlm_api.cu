@@ -129,6 +129,16 @@ int* device_error_word() {
 
 }  // namespace dlm
 
+namespace {
+
+// Every kernel records device-side failures in the error word; refuse to launch without it.
+int require_error_word() {
+  if (!dlm::device_error_word()) return dlm::fail(DLM_ERR_CUDA, "device error word unavailable on this device");
+  return DLM_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 int dlm_version(void) { return DLM_VERSION_MAJOR * 10000 + DLM_VERSION_MINOR * 100 + DLM_VERSION_PATCH; }
@@ -230,14 +240,21 @@ int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v
         if ((t->stride[i] * 2) % 16 != 0 || t->stride[i] * 2 >= (1LL << 40))
           return fail(DLM_ERR_ALIGN, "bf16 attention needs strides that are multiples of 16 bytes");
     }
+    if ((st = require_error_word())) return st;
     return dlm::launch_attn_tc_bf16(a, t_stream);
   }
+  if ((st = require_error_word())) return st;
   return dlm::launch_attn_f32(a, t_stream);
 }
 
-int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse) {
+}  // extern "C"
+
+namespace {
+
+// Validates the arguments of the vocabulary reduction and fills *a.
+int prepare_vocab(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
+                  dlm::VocabArgs* a) {
   using dlm::fail;
-  t_last_error[0] = '\0';
   int st;
   if ((st = check_tensor(logits, "logits", kMaskBF16F32, 2, 3))) return st;
   if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 1, 3))) return st;
@@ -261,24 +278,22 @@ int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tenso
   }
   if (overlaps(argmax, conf) || overlaps(argmax, lse) || overlaps(conf, lse))
     return fail(DLM_ERR_ARG, "outputs overlap each other");
-  if (N == 0) return DLM_OK;
-  dlm::VocabArgs a;
-  a.logits = logits->data;
-  a.is_bf16 = logits->dtype == DLM_BF16;
-  a.N = N;
-  a.V = V;
-  a.row_stride = N > 1 ? row_stride : V;
-  a.argmax = static_cast<int32_t*>(argmax->data);
-  a.conf = static_cast<float*>(conf->data);
-  a.lse = static_cast<float*>(lse->data);
-  return dlm::launch_vocab_confidence(a, t_stream);
+  a->logits = logits->data;
+  a->is_bf16 = logits->dtype == DLM_BF16;
+  a->N = N;
+  a->V = V;
+  a->row_stride = N > 1 ? row_stride : V;
+  a->argmax = static_cast<int32_t*>(argmax->data);
+  a->conf = static_cast<float*>(conf->data);
+  a->lse = static_cast<float*>(lse->data);
+  return DLM_OK;
 }
 
-int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
-                      const dlm_tensor* conf, const dlm_refine_params* params, dlm_tensor* new_tokens,
-                      dlm_tensor* new_mask, dlm_tensor* n_edits) {
+// Validates the arguments of the refine update and fills *a.
+int prepare_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax, const dlm_tensor* conf,
+                   const dlm_refine_params* params, dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits,
+                   dlm::UpdateArgs* a) {
   using dlm::fail;
-  t_last_error[0] = '\0';
   int st;
   if ((st = check_tensor(tokens, "tokens", 1 << DLM_I32, 2, 2))) return st;
   if ((st = check_tensor(mask, "mask", 1 << DLM_U8, 2, 2))) return st;
@@ -294,6 +309,10 @@ int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dl
     if (t->shape[0] != B || t->shape[1] != L) return fail(DLM_ERR_SHAPE, "all [B, L] tensors must share B and L");
   if (n_edits->shape[0] != B) return fail(DLM_ERR_SHAPE, "n_edits must have B entries");
   if (L > (1 << 24)) return fail(DLM_ERR_SHAPE, "L too large (max 2^24)");
+  if (B > 0 && (!params->prompt_lens || !params->seq_lens))
+    return fail(DLM_ERR_NULL, "params: prompt_lens / seq_lens is NULL");
+  if (reinterpret_cast<uintptr_t>(params->prompt_lens) % 4 != 0 || reinterpret_cast<uintptr_t>(params->seq_lens) % 4 != 0)
+    return fail(DLM_ERR_ALIGN, "params: prompt_lens / seq_lens not 4-byte aligned");
   if (std::isnan(params->edit_threshold)) return fail(DLM_ERR_ARG, "edit_threshold is NaN");
   if (params->remask_k < 0 && !(params->remask_frac >= 0.f && params->remask_frac <= 1.f))
     return fail(DLM_ERR_ARG, "remask_frac must be in [0, 1] when remask_k < 0");
@@ -311,30 +330,111 @@ int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dl
     }
   if (overlaps(new_tokens, new_mask) || overlaps(new_tokens, n_edits) || overlaps(new_mask, n_edits))
     return fail(DLM_ERR_ARG, "outputs overlap each other");
-  if (B == 0) return DLM_OK;
+  a->tokens = static_cast<const int32_t*>(tokens->data);
+  a->mask = static_cast<const uint8_t*>(mask->data);
+  a->argmax = static_cast<const int32_t*>(argmax->data);
+  a->conf = static_cast<const float*>(conf->data);
+  a->new_tokens = static_cast<int32_t*>(new_tokens->data);
+  a->new_mask = static_cast<uint8_t*>(new_mask->data);
+  a->n_edits = static_cast<int32_t*>(n_edits->data);
+  a->s_tokens = tokens->stride[0];
+  a->s_mask = mask->stride[0];
+  a->s_argmax = argmax->stride[0];
+  a->s_conf = conf->stride[0];
+  a->s_new_tokens = new_tokens->stride[0];
+  a->s_new_mask = new_mask->stride[0];
+  a->B = static_cast<int>(B);
+  a->L = static_cast<int>(L);
+  a->edit_threshold = params->edit_threshold;
+  a->remask_k = params->remask_k;
+  a->remask_frac = params->remask_frac;
+  a->mask_id = params->mask_id;
+  a->prompt_lens = params->prompt_lens;
+  a->seq_lens = params->seq_lens;
+  return DLM_OK;
+}
+
+// Validates the fused step's arguments (both parts plus their coupling).
+int prepare_step(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* mask,
+                 const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
+                 dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits, dlm::VocabArgs* va,
+                 dlm::UpdateArgs* ua) {
+  using dlm::fail;
+  int st;
+  if ((st = prepare_vocab(logits, argmax, conf, lse, va))) return st;
+  if ((st = prepare_update(tokens, mask, argmax, conf, params, new_tokens, new_mask, n_edits, ua))) return st;
+  if (va->N != static_cast<int64_t>(ua->B) * ua->L)
+    return fail(DLM_ERR_SHAPE, "logits must have one row per (sequence, position): B * L rows");
+  if (logits->ndim == 3 && (logits->shape[0] != ua->B || logits->shape[1] != ua->L))
+    return fail(DLM_ERR_SHAPE, "3-D logits must be [B, L, V]");
+  if (!is_dense(argmax) || !is_dense(conf)) return fail(DLM_ERR_STRIDE, "argmax and conf must be contiguous [B, L]");
+  const dlm_tensor* ins[3] = {tokens, mask, logits};
+  const dlm_tensor* outs[6] = {argmax, conf, lse, new_tokens, new_mask, n_edits};
+  for (int o = 0; o < 6; ++o)
+    for (int i = 0; i < 3; ++i) {
+      if ((o == 3 && i == 0) || (o == 4 && i == 1)) continue;  // in-place update allowed
+      if (overlaps(outs[o], ins[i])) return fail(DLM_ERR_ARG, "an output overlaps an input");
+    }
+  for (int o = 0; o < 3; ++o)
+    for (int q = 3; q < 6; ++q)
+      if (overlaps(outs[o], outs[q])) return fail(DLM_ERR_ARG, "outputs overlap each other");
+  return DLM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse) {
+  t_last_error[0] = '\0';
+  dlm::VocabArgs a;
+  int st = prepare_vocab(logits, argmax, conf, lse, &a);
+  if (st != DLM_OK || a.N == 0) return st;
+  if ((st = require_error_word())) return st;
+  return dlm::launch_vocab_confidence(a, t_stream);
+}
+
+int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
+                      const dlm_tensor* conf, const dlm_refine_params* params, dlm_tensor* new_tokens,
+                      dlm_tensor* new_mask, dlm_tensor* n_edits) {
+  t_last_error[0] = '\0';
   dlm::UpdateArgs a;
-  a.tokens = static_cast<const int32_t*>(tokens->data);
-  a.mask = static_cast<const uint8_t*>(mask->data);
-  a.argmax = static_cast<const int32_t*>(argmax->data);
-  a.conf = static_cast<const float*>(conf->data);
-  a.new_tokens = static_cast<int32_t*>(new_tokens->data);
-  a.new_mask = static_cast<uint8_t*>(new_mask->data);
-  a.n_edits = static_cast<int32_t*>(n_edits->data);
-  a.s_tokens = tokens->stride[0];
-  a.s_mask = mask->stride[0];
-  a.s_argmax = argmax->stride[0];
-  a.s_conf = conf->stride[0];
-  a.s_new_tokens = new_tokens->stride[0];
-  a.s_new_mask = new_mask->stride[0];
-  a.B = static_cast<int>(B);
-  a.L = static_cast<int>(L);
-  a.edit_threshold = params->edit_threshold;
-  a.remask_k = params->remask_k;
-  a.remask_frac = params->remask_frac;
-  a.mask_id = params->mask_id;
-  a.prompt_lens = params->prompt_lens;
-  a.seq_lens = params->seq_lens;
+  int st = prepare_update(tokens, mask, argmax, conf, params, new_tokens, new_mask, n_edits, &a);
+  if (st != DLM_OK || a.B == 0) return st;
+  if ((st = require_error_word())) return st;
   return dlm::launch_refine_update(a, t_stream);
+}
+
+size_t dlm_refine_step_workspace_bytes(int64_t batch) {
+  return batch > 0 ? static_cast<size_t>(batch) * sizeof(int32_t) : 0;
+}
+
+int dlm_refine_step(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* mask,
+                    const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
+                    dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits, void* workspace,
+                    size_t workspace_bytes) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  dlm::VocabArgs va;
+  dlm::UpdateArgs ua;
+  int st = prepare_step(logits, tokens, mask, params, argmax, conf, lse, new_tokens, new_mask, n_edits, &va, &ua);
+  if (st != DLM_OK) return st;
+  if (ua.B == 0 || va.N == 0) return DLM_OK;
+  if (!workspace) return fail(DLM_ERR_NULL, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) % 4 != 0) return fail(DLM_ERR_ALIGN, "workspace not 4-byte aligned");
+  if (workspace_bytes < dlm_refine_step_workspace_bytes(ua.B))
+    return fail(DLM_ERR_ARG, "workspace too small: %zu bytes, %zu needed", workspace_bytes,
+                dlm_refine_step_workspace_bytes(ua.B));
+  const uintptr_t wlo = reinterpret_cast<uintptr_t>(workspace);
+  const uintptr_t whi = wlo + dlm_refine_step_workspace_bytes(ua.B);
+  const dlm_tensor* all[9] = {logits, tokens, mask, argmax, conf, lse, new_tokens, new_mask, n_edits};
+  for (const dlm_tensor* t : all) {
+    uintptr_t lo, hi;
+    byte_span(t, &lo, &hi);
+    if (numel(t) > 0 && lo < whi && wlo < hi) return fail(DLM_ERR_ARG, "workspace overlaps a tensor");
+  }
+  if ((st = require_error_word())) return st;
+  return dlm::launch_vocab_step(va, ua, static_cast<int*>(workspace), t_stream);
 }
 
 }  // extern "C"

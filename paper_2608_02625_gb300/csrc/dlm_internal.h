@@ -60,4 +60,8 @@ struct UpdateArgs {
 
 int launch_refine_update(const UpdateArgs& a, cudaStream_t stream);
 
+// Fused vocabulary reduction + update (rows of sequence b are b * L .. b * L + L - 1;
+// u.argmax / u.conf alias a.argmax / a.conf). counters: int32[B], zero on entry.
+int launch_vocab_step(const VocabArgs& a, const UpdateArgs& u, int* counters, cudaStream_t stream);
+
 }  // namespace dlm

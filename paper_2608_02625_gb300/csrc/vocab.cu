@@ -11,7 +11,11 @@
 // 16-byte vector raises the running maximum. Threads combine by warp shuffles,
 // warps through shared memory, and -- when there are too few rows to fill the
 // GPU -- the CTAs of a thread-block cluster that split one row combine through
-// distributed shared memory. No global scratch memory.
+// distributed shared memory (no global scratch memory).
+//
+// The fused variant (vocab_step_kernel) also runs step A3: the CTA finishing a
+// sequence's last row performs its update, counted with one int32 arrival
+// counter per sequence in caller-provided scratch memory.
 #include <cooperative_groups.h>
 
 #include <cmath>
@@ -19,6 +23,7 @@
 
 #include "dlm_common.cuh"
 #include "dlm_internal.h"
+#include "update_impl.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -211,6 +216,37 @@ __global__ void __launch_bounds__(kThreads, 4) vocab_rows_kernel(VocabArgs a) {
   }
 }
 
+// Fused A2 + A3: one CTA per row as above; the CTA that completes the last
+// row of a sequence (an arrival counter per sequence in `counters`) then runs
+// that sequence's refine update, reading the predictions the other CTAs wrote
+// around L1. The counter of a sequence is returned to zero by its last CTA,
+// so `counters` must be zero before the first launch and is zero after each
+// complete launch.
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kThreads, 4) vocab_step_kernel(VocabArgs a, UpdateArgs u, int* counters, int* err) {
+  __shared__ UpdateShared<kThreads> ush;
+  __shared__ int last;
+  const int esz = BF16 ? 2 : 4;
+  for (int64_t rowi = blockIdx.x; rowi < a.N; rowi += gridDim.x) {
+    const char* row = static_cast<const char*>(a.logits) + rowi * a.row_stride * esz;
+    Partial p = scan_range<BF16, VEC>(row, 0, a.V);
+    p = block_reduce(p);
+    const int b = static_cast<int>(rowi / u.L);
+    if (threadIdx.x == 0) {
+      write_out(a, rowi, p);
+      __threadfence();  // the predictions are visible before the arrival is
+      last = atomicAdd(&counters[b], 1) == u.L - 1;
+    }
+    __syncthreads();
+    if (last) {
+      if (threadIdx.x == 0) counters[b] = 0;
+      __threadfence();
+      refine_sequence<kThreads, true>(u, b, err, ush);
+    }
+    __syncthreads();
+  }
+}
+
 // A cluster of `csize` CTAs per row; CTA c scans a contiguous chunk, rank 0
 // combines the chunk partials through distributed shared memory.
 template <bool BF16, bool VEC>
@@ -294,6 +330,28 @@ int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream) {
   const bool vec = (reinterpret_cast<uintptr_t>(a.logits) % 16 == 0) && ((a.row_stride * esz) % 16 == 0);
   if (a.is_bf16) return vec ? launch_typed<true, true>(a, stream) : launch_typed<true, false>(a, stream);
   return vec ? launch_typed<false, true>(a, stream) : launch_typed<false, false>(a, stream);
+}
+
+int launch_vocab_step(const VocabArgs& a, const UpdateArgs& u, int* counters, cudaStream_t stream) {
+  if (a.N == 0) return DLM_OK;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t cap = 2LL * 64 * sms;
+  const unsigned grid = static_cast<unsigned>(a.N < cap ? a.N : cap);
+  const int esz = a.is_bf16 ? 2 : 4;
+  const bool vec = (reinterpret_cast<uintptr_t>(a.logits) % 16 == 0) && ((a.row_stride * esz) % 16 == 0);
+  int* err = device_error_word();
+  if (a.is_bf16) {
+    if (vec) vocab_step_kernel<true, true><<<grid, kThreads, 0, stream>>>(a, u, counters, err);
+    else vocab_step_kernel<true, false><<<grid, kThreads, 0, stream>>>(a, u, counters, err);
+  } else {
+    if (vec) vocab_step_kernel<false, true><<<grid, kThreads, 0, stream>>>(a, u, counters, err);
+    else vocab_step_kernel<false, false><<<grid, kThreads, 0, stream>>>(a, u, counters, err);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "refine_step launch: %s", cudaGetErrorString(e));
+  return DLM_OK;
 }
 
 }  // namespace dlm

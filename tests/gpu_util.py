@@ -53,6 +53,20 @@ def host_logit_rows(w: Workload, step: int, rows, tokens=None, mask=None) -> np.
     return x
 
 
+def check_update_margin(gpu, ref, amb, where=""):
+    """Decision-margin parity of the update: GPU (tokens, mask, n_edits) against
+    the oracle's, computed from the oracle's own vocabulary outputs. They must be
+    identical at every position outside `amb`, and n_edits identical for every
+    sequence without an ambiguous position."""
+    g_tok, g_msk, g_ne = gpu
+    diff = (g_tok != ref[0]) | (g_msk != ref[1])
+    assert not np.any(diff & ~amb), f"{where}: update differs at unambiguous positions {np.argwhere(diff & ~amb)[:8]}"
+    for b in range(g_tok.shape[0]):
+        if not amb[b].any():
+            assert g_ne[b] == ref[2][b], f"{where}: n_edits of sequence {b}"
+    return int(amb.sum())
+
+
 def check_vocab(am_gpu, conf_gpu, lse_gpu, am_ref, conf_ref, lse_ref, where=""):
     am_gpu, conf_gpu, lse_gpu = (np.asarray(a) for a in (am_gpu, conf_gpu, lse_gpu))
     bad = np.nonzero(am_gpu != am_ref)[0]
@@ -68,8 +82,14 @@ def ambiguous_positions(w: Workload, step: int, conf_ref: np.ndarray, state, arg
     """Positions where a decision of the update is within the conf tolerance of
     its boundary: |conf - tau| within CONF_RTOL, or conf within CONF_RTOL of the
     k-th smallest response conf. Returns a bool [B, L] array."""
+    return ambiguous_for(w.edit_threshold[step], w.remask_k, w.remask_frac, conf_ref, state, argmax_ref, prompt,
+                         seqlen)
+
+
+def ambiguous_for(edit_threshold, remask_k, remask_frac, conf_ref, state, argmax_ref, prompt, seqlen):
+    """ambiguous_positions for explicit update parameters."""
     tok, msk = state
-    tau = np.float32(w.edit_threshold[step])
+    tau = np.float32(edit_threshold)
     B, L = tok.shape
     amb = np.zeros((B, L), dtype=bool)
     for b in range(B):
@@ -78,7 +98,7 @@ def ambiguous_positions(w: Workload, step: int, conf_ref: np.ndarray, state, arg
         tol = CONF_RTOL * np.maximum(c, 1e-30) * 2
         edit_cand = (msk[b, p:n] == 0) & (argmax_ref[b, p:n] != tok[b, p:n])
         amb[b, p:n] |= edit_cand & (np.abs(c - float(tau)) <= tol)
-        k = remask_count(w.remask_k, w.remask_frac, n - p)
+        k = remask_count(remask_k, remask_frac, n - p)
         if 0 < k < n - p:
             kth = np.sort(c)[k - 1]
             amb[b, p:n] |= np.abs(c - kth) <= CONF_RTOL * max(kth, 1e-30) * 2

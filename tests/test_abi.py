@@ -153,6 +153,7 @@ def P(**kw):
 @pytest.mark.parametrize("case,status", [
     ("null_params", -1), ("nan_threshold", -6), ("frac_above_one", -6), ("frac_nan", -6), ("mask_dtype", -2),
     ("shape_mismatch", -3), ("n_edits_shape", -3), ("partial_alias", -6), ("output_overlaps_input", -6),
+    ("null_prompt_lens", -1), ("null_seq_lens", -1), ("misaligned_seq_lens", -5),
 ])
 def test_update_rejects(case, status):
     if case == "null_params":
@@ -173,6 +174,12 @@ def test_update_rejects(case, status):
         assert update(P(), nt=T(I32, [2, 8], 1 * MB + 4)) == status
     elif case == "output_overlaps_input":
         assert update(P(), nt=T(I32, [2, 8], 4 * MB)) == status
+    elif case == "null_prompt_lens":
+        assert update(P(prompt_lens=None)) == status
+    elif case == "null_seq_lens":
+        assert update(P(seq_lens=None)) == status
+    elif case == "misaligned_seq_lens":
+        assert update(P(seq_lens=9 * MB + 2)) == status
 
 
 def test_last_error_message():
@@ -180,3 +187,51 @@ def test_last_error_message():
     q, k, v, sl, o = good_attn(D=96)
     assert attn(q, k, v, sl, o) == -3
     assert b"head_dim" in lib.dlm_last_error()
+
+
+def step(params, ws=10 * MB, ws_bytes=8, **over):
+    from paper_2608_02625_gb300.binding import lib
+    d = dict(lg=T(BF16, [16, 1000], 11 * MB), tok=T(I32, [2, 8], 1 * MB), msk=T(U8, [2, 8], 2 * MB),
+             am=T(I32, [2, 8], 3 * MB), cf=T(F32, [2, 8], 4 * MB), ls=T(F32, [2, 8], 12 * MB),
+             nt=T(I32, [2, 8], 5 * MB), nm=T(U8, [2, 8], 6 * MB), ne=T(I32, [2], 7 * MB))
+    d.update(over)
+    r = lambda x: ctypes.byref(x) if x is not None else None
+    return lib.dlm_refine_step(r(d["lg"]), r(d["tok"]), r(d["msk"]), ctypes.byref(params) if params else None,
+                               r(d["am"]), r(d["cf"]), r(d["ls"]), r(d["nt"]), r(d["nm"]), r(d["ne"]),
+                               ctypes.c_void_p(ws), ctypes.c_size_t(ws_bytes))
+
+
+def test_step_workspace_bytes():
+    from paper_2608_02625_gb300.binding import lib
+    assert [lib.dlm_refine_step_workspace_bytes(b) for b in (0, 1, 32, -3)] == [0, 4, 128, 0]
+
+
+@pytest.mark.parametrize("case,status", [
+    ("null_params", -1), ("null_workspace", -1), ("workspace_small", -6), ("workspace_misaligned", -5),
+    ("rows_not_BL", -3), ("logits_3d_mismatch", -3), ("strided_conf", -4), ("lse_overlaps_new_tokens", -6),
+    ("argmax_overlaps_tokens", -6), ("nan_threshold", -6), ("workspace_overlaps_lse", -6),
+])
+def test_step_rejects(case, status):
+    if case == "null_params":
+        assert step(None) == status
+    elif case == "null_workspace":
+        assert step(P(), ws=0) == status
+    elif case == "workspace_small":
+        assert step(P(), ws_bytes=7) == status
+    elif case == "workspace_misaligned":
+        assert step(P(), ws=10 * MB + 2) == status
+    elif case == "rows_not_BL":
+        assert step(P(), lg=T(BF16, [15, 1000], 11 * MB),
+                    am=T(I32, [15], 3 * MB), cf=T(F32, [15], 4 * MB), ls=T(F32, [15], 12 * MB)) == status
+    elif case == "logits_3d_mismatch":
+        assert step(P(), lg=T(BF16, [4, 4, 1000], 11 * MB)) == status
+    elif case == "strided_conf":
+        assert step(P(), cf=T(F32, [2, 8], 4 * MB, strides=[16, 1])) == status
+    elif case == "lse_overlaps_new_tokens":
+        assert step(P(), ls=T(F32, [2, 8], 5 * MB + 8)) == status
+    elif case == "argmax_overlaps_tokens":
+        assert step(P(), am=T(I32, [2, 8], 1 * MB)) == status
+    elif case == "nan_threshold":
+        assert step(P(edit_threshold=math.nan)) == status
+    elif case == "workspace_overlaps_lse":
+        assert step(P(), ws=12 * MB + 60) == status
