@@ -19,7 +19,8 @@
  * - Tensors are passed as dlm_tensor descriptors: a DEVICE pointer of the
  *   current CUDA device, a dtype, the shape and the strides in elements.
  *   The caller owns every buffer; the library allocates no device memory and
- *   keeps no pointer after a call returns.
+ *   keeps no pointer after a call returns. Its only device memory is static:
+ *   the error word and the 16 KB scratch of dlm_refine_step_static.
  * - Calls are asynchronous on the stream set by dlm_set_stream for the calling
  *   thread (default: the legacy default stream). Outputs are valid once that
  *   stream has been synchronised. Arguments are validated on the host before
@@ -191,6 +192,40 @@ int dlm_refine_step(const dlm_tensor* logits, const dlm_tensor* tokens, const dl
                     dlm_tensor* n_edits, void* workspace, size_t workspace_bytes);
 /* Bytes of workspace dlm_refine_step needs for a batch of `batch` sequences. */
 size_t dlm_refine_step_workspace_bytes(int64_t batch);
+
+/* Largest batch dlm_refine_step_static accepts (its static scratch: 16 KB). */
+#define DLM_STATIC_STEP_MAX_BATCH 4096
+
+/*
+ * dlm_refine_step without a workspace argument; the paper has no counterpart
+ * (it is a deployment convenience of this library, not part of the method).
+ * For callers that cannot allocate device memory: a serving engine whose
+ * allocator reserves nearly all of HBM up front (a cudaMalloc outside its pool
+ * fails or fragments it), a latency-critical loop that cannot take
+ * cudaMalloc's implicit device synchronisation, or a plugin interface with a
+ * fixed signature and no slot for a workspace.
+ *
+ * Computes exactly what dlm_refine_step computes, with the same arguments
+ * minus the workspace. The per-sequence counters live in a static device
+ * array of DLM_STATIC_STEP_MAX_BATCH int32 inside the library, which every
+ * device that loads the library holds until the process exits. The call
+ * allocates nothing (no cudaMalloc, cudaFree or allocating library routine).
+ *
+ * - The first call on a device sets up that device: it takes the array's
+ *   device address with cudaGetSymbolAddress, with that device current.
+ *   Make that first call before any stream capture on the device.
+ * - Each call clears the counters it uses (an asynchronous memset on the
+ *   call's stream) and then launches the fused kernel.
+ * - All calls on one device share the array: calls that overlap on the GPU
+ *   (different streams, or different host threads) race on it and give
+ *   undefined results. Issue them on one stream.
+ * - B > DLM_STATIC_STEP_MAX_BATCH returns DLM_ERR_SHAPE with nothing
+ *   launched; use dlm_refine_step with a workspace for larger batches.
+ */
+int dlm_refine_step_static(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* mask,
+                           const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf,
+                           dlm_tensor* lse, dlm_tensor* new_tokens, dlm_tensor* new_mask,
+                           dlm_tensor* n_edits);
 
 /* Sets the CUDA stream (a cudaStream_t) used by later calls on this thread. */
 int dlm_set_stream(void* stream);

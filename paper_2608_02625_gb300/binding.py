@@ -50,10 +50,11 @@ def _load():
     lib.dlm_refine_update.argtypes = [P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
     lib.dlm_refine_step.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P,
                                     ctypes.c_void_p, ctypes.c_size_t]
+    lib.dlm_refine_step_static.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P]
     lib.dlm_refine_step_workspace_bytes.argtypes = [ctypes.c_int64]
     lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
-    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step", "dlm_set_stream",
-              "dlm_version", "dlm_get_device_error"):
+    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
+              "dlm_refine_step_static", "dlm_set_stream", "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
     lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
     lib.dlm_get_stream.restype = ctypes.c_void_p
@@ -181,6 +182,21 @@ def dlm_refine_step(logits, tokens, mask, params: RefineParams, argmax, conf, ls
     nbytes = workspace.numel() * workspace.element_size()
     _check(lib.dlm_refine_step(*[_ref(d) for d in ins], ctypes.byref(cp), *[_ref(d) for d in outs],
                                ctypes.c_void_p(workspace.data_ptr() if nbytes else None), ctypes.c_size_t(nbytes)))
+    return argmax, conf, lse, new_tokens, new_mask, n_edits
+
+
+def dlm_refine_step_static(logits, tokens, mask, params: RefineParams, argmax, conf, lse, new_tokens, new_mask,
+                           n_edits):
+    """dlm_refine_step with the library's static scratch instead of a workspace,
+    for callers that cannot allocate device memory. The first call on a device
+    sets that device up (make it before any stream capture); calls that overlap
+    on the GPU race on the shared scratch."""
+    _prepare(logits, tokens, mask, argmax, conf, lse, new_tokens, new_mask, n_edits, params.prompt_lens,
+             params.seq_lens)
+    ins = [describe(t) for t in (logits, tokens, mask)]
+    outs = [describe(t) for t in (argmax, conf, lse, new_tokens, new_mask, n_edits)]
+    cp = params.to_c()
+    _check(lib.dlm_refine_step_static(*[_ref(d) for d in ins], ctypes.byref(cp), *[_ref(d) for d in outs]))
     return argmax, conf, lse, new_tokens, new_mask, n_edits
 
 

@@ -438,3 +438,76 @@ int dlm_refine_step(const dlm_tensor* logits, const dlm_tensor* tokens, const dl
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// dlm_refine_step_static: the fused step with library-owned scratch memory.
+//
+// For callers that cannot allocate device memory themselves: a serving engine
+// whose allocator reserves nearly all of HBM for weights and KV cache up front
+// (a cudaMalloc outside that pool fails or fragments it), a latency-critical
+// loop that cannot afford cudaMalloc's implicit device synchronisation, or a
+// plugin interface whose fixed signature has no slot for a workspace. Instead
+// of a caller-provided workspace, the per-sequence arrival counters live in
+// the file-scope array below: DLM_STATIC_STEP_MAX_BATCH int32 values (16 KB),
+// held by every device that loads the library until the process exits.
+//
+// On the host, g_dlm_step_scratch is only a stand-in for the device symbol:
+// its device address is taken once per device, with that device current, by
+// cudaGetSymbolAddress on the first call on that device, and that address is
+// what the kernel receives. Every call on a device shares the array and finds
+// the last call's contents there, so each call clears the counters it uses
+// (cudaMemsetAsync on the caller's stream) before the launch; two calls that
+// overlap on the GPU race on the counters.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) int32_t g_dlm_step_scratch[DLM_STATIC_STEP_MAX_BATCH];
+
+namespace {
+
+std::mutex g_scratch_mu;
+int32_t* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_dlm_step_scratch on the current device (set up on first use).
+int static_step_scratch(int32_t** out) {
+  using dlm::fail;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return fail(DLM_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_dlm_step_scratch);
+    if (e != cudaSuccess)
+      return fail(DLM_ERR_CUDA, "cudaGetSymbolAddress(static step scratch): %s", cudaGetErrorString(e));
+    g_scratch_addr[dev] = static_cast<int32_t*>(ptr);
+  }
+  *out = g_scratch_addr[dev];
+  return DLM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dlm_refine_step_static(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* mask,
+                           const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
+                           dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  dlm::VocabArgs va;
+  dlm::UpdateArgs ua;
+  int st = prepare_step(logits, tokens, mask, params, argmax, conf, lse, new_tokens, new_mask, n_edits, &va, &ua);
+  if (st != DLM_OK) return st;
+  if (ua.B == 0 || va.N == 0) return DLM_OK;
+  if (ua.B > DLM_STATIC_STEP_MAX_BATCH)
+    return fail(DLM_ERR_SHAPE, "batch %d exceeds the static scratch maximum of %d sequences (use dlm_refine_step)",
+                ua.B, DLM_STATIC_STEP_MAX_BATCH);
+  if ((st = require_error_word())) return st;
+  int32_t* counters = nullptr;
+  if ((st = static_step_scratch(&counters))) return st;
+  cudaError_t e = cudaMemsetAsync(counters, 0, static_cast<size_t>(ua.B) * sizeof(int32_t), t_stream);
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "clearing the static step scratch: %s", cudaGetErrorString(e));
+  return dlm::launch_vocab_step(va, ua, counters, t_stream);
+}
+
+}  // extern "C"

@@ -235,3 +235,16 @@ def test_step_rejects(case, status):
         assert step(P(edit_threshold=math.nan)) == status
     elif case == "workspace_overlaps_lse":
         assert step(P(), ws=12 * MB + 60) == status
+
+
+def test_static_step_rejects_batch_above_maximum_on_the_host():
+    from paper_2608_02625_gb300.binding import lib
+    B = 4097
+    d = dict(lg=T(BF16, [B, 16], 11 * MB), tok=T(I32, [B, 1], 1 * MB), msk=T(U8, [B, 1], 2 * MB),
+             am=T(I32, [B, 1], 3 * MB), cf=T(F32, [B, 1], 4 * MB), ls=T(F32, [B, 1], 12 * MB),
+             nt=T(I32, [B, 1], 5 * MB), nm=T(U8, [B, 1], 6 * MB), ne=T(I32, [B], 7 * MB))
+    r = ctypes.byref
+    st = lib.dlm_refine_step_static(r(d["lg"]), r(d["tok"]), r(d["msk"]), r(P()), r(d["am"]), r(d["cf"]),
+                                    r(d["ls"]), r(d["nt"]), r(d["nm"]), r(d["ne"]))
+    assert st == -3
+    assert b"4096" in lib.dlm_last_error()
