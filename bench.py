@@ -264,6 +264,90 @@ def job_steps_per_s(ms_per_step: float, world: int) -> float:
 
 # ---------------------------------------------------------------- GPU arm
 
+def measure_loop(args, w, Bn, q, k, v, out, logits, tok0, msk0, params, seqlen, stream):
+    """Refine passes on one resident batch with tokens / mask updated in place,
+    until no confident edit remains or --loop-steps passes have run: (a) as one
+    launch of a recorded loop, (b) pass by pass with n_edits read back by the
+    host after each pass. Both run the same passes on the same buffers."""
+    import torch
+    d = tok0.device
+    tok, msk = tok0.clone(), msk0.clone()
+    am = torch.empty((w.B, w.L), dtype=torch.int32, device=d)
+    cf = torch.empty((w.B, w.L), dtype=torch.float32, device=d)
+    ls = torch.empty((w.B, w.L), dtype=torch.float32, device=d)
+    ne = torch.zeros(w.B, dtype=torch.int32, device=d)
+    ws = torch.zeros(w.B, dtype=torch.int32, device=d)
+    steps = torch.zeros(1, dtype=torch.int32, device=d)
+
+    def one_pass():
+        Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+        if args.path == "fused":
+            Bn.dlm_refine_step(logits, tok, msk, params, am, cf, ls, tok, msk, ne, ws)
+        else:
+            Bn.dlm_vocab_confidence(logits, am.view(-1), cf.view(-1), ls.view(-1))
+            Bn.dlm_refine_update(tok, msk, am, cf, params, tok, msk, ne)
+
+    def host_driven():
+        n = 0
+        for s in range(args.loop_steps):
+            one_pass()
+            n = s + 1
+            if not bool((ne > 0).any()):   # host round trip after every pass
+                break
+        return n
+
+    side = torch.cuda.Stream(d)
+    side.wait_stream(stream)
+    with torch.cuda.stream(side):
+        Bn.dlm_loop_begin(steps)
+        try:
+            one_pass()
+        except BaseException:
+            Bn.dlm_loop_cancel()
+            raise
+        loop = Bn.dlm_loop_end(ne, args.loop_steps, steps)
+    torch.cuda.synchronize()
+    reps = 10
+    try:
+        with torch.cuda.stream(side):
+            for _ in range(3):
+                tok.copy_(tok0)
+                msk.copy_(msk0)
+                loop.launch()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t_graph = 0.0
+            for _ in range(reps):
+                tok.copy_(tok0)
+                msk.copy_(msk0)
+                e0.record(side)
+                loop.launch()
+                e1.record(side)
+                torch.cuda.synchronize()
+                t_graph += e0.elapsed_time(e1)
+            passes = int(steps.item())
+            graph_state = (tok.clone(), msk.clone())
+            t_host = 0.0
+            for r in range(reps + 1):
+                tok.copy_(tok0)
+                msk.copy_(msk0)
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                n_host = host_driven()
+                torch.cuda.synchronize()
+                if r > 0:   # the first run warms up
+                    t_host += (time.perf_counter() - t0) * 1e3
+            same = bool(torch.equal(tok, graph_state[0]) and torch.equal(msk, graph_state[1]))
+    finally:
+        loop.close()
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the loop measurement")
+    return {"workload": w.name, "max_passes": args.loop_steps, "passes": passes, "passes_host_driven": n_host,
+            "same_result": same, "ms_graph_launch": t_graph / reps, "ms_host_driven": t_host / reps,
+            "note": "pass = attention + vocabulary reduction + in-place update on resident q/k/v and logits; "
+                    "graph: CUDA events around one launch; host-driven: wall clock, one n_edits read-back per pass"}
+
+
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -402,6 +486,12 @@ def run_ours(args, rank, world):
     if rank != 0:
         return None
 
+    # ---- multi-pass refinement: the recorded pass repeated by one graph launch
+    # (device-side early stop) against the same passes driven from the host
+    loop_info = None
+    if args.loop_steps > 0:
+        loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
+
     attn_flops = w.attn_flops()
     vocab_bytes = w.vocab_bytes()
     kern = {
@@ -446,6 +536,7 @@ def run_ours(args, rank, world):
         "gpu_launches": (2 if fused else 3) * args.steps,
         "path": args.path,
         "e2e": e2e,
+        "loop": loop_info,
     }
     if timer is not None:
         res["cpu_baseline"] = timer.run()
@@ -490,6 +581,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--loop-steps", type=int, default=4,
+                    help="also time a recorded multi-pass loop with device-side early stop (0: skip)")
     ap.add_argument("--path", default="separate", choices=["fused", "separate"],
                     help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
                          "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")

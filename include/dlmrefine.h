@@ -12,7 +12,8 @@
  *   dlm_refine_update     commit masked positions, edit confident changes,
  *                         remask the k least confident positions
  *
- * dlm_refine_step does the last two in one launch (same results).
+ * dlm_refine_step does the last two in one launch (same results), and
+ * dlm_loop_* repeat a recorded pass on the GPU until no confident edit remains.
  *
  * Conventions shared by every call
  * --------------------------------
@@ -226,6 +227,42 @@ int dlm_refine_step_static(const dlm_tensor* logits, const dlm_tensor* tokens, c
                            const dlm_refine_params* params, dlm_tensor* argmax, dlm_tensor* conf,
                            dlm_tensor* lse, dlm_tensor* new_tokens, dlm_tensor* new_mask,
                            dlm_tensor* n_edits);
+
+/*
+ * Multi-pass refinement as one graph launch, with the early stop on the device
+ * (passes repeat until no confident edit remains, Appendix C.4 / Table 11).
+ *
+ *   int32_t* steps;                  // device int32: passes run by a launch
+ *   dlm_loop_begin(steps);           // start recording one pass
+ *   ... the pass: the caller's model forward, dlm_bidir_attn,
+ *       dlm_refine_step (or the two separate calls) on the same stream ...
+ *   dlm_loop_end(n_edits, B, max_steps, &loop);
+ *   dlm_loop_launch(loop);           // runs the recorded pass repeatedly
+ *   dlm_loop_destroy(loop);
+ *
+ * dlm_loop_begin starts a stream capture (thread-local mode) on the calling
+ * thread's stream, which must be a created stream (not the legacy default):
+ * calls issued on it until dlm_loop_end are recorded, not run. The recorded
+ * pass must read its inputs from and write its outputs to fixed device
+ * buffers (in-place token update: new_tokens / new_mask aliasing tokens /
+ * mask), because every repetition replays the same launches.
+ *
+ * dlm_loop_end builds a CUDA graph: steps = 0, then WHILE { pass; steps += 1;
+ * continue iff steps < max_steps and n_edits[b] > 0 for some b < B and the
+ * device error word is clear }. n_edits is the [B] int32 edit count written
+ * by the recorded pass. The test runs on the GPU after each pass, so there is
+ * no host round trip between passes. Validation failures and capture errors
+ * end the capture and return an error; dlm_loop_cancel ends an unfinished
+ * recording. A loop may be launched any number of times (on the calling
+ * thread's stream); each launch restarts steps at 0. The loop keeps device
+ * pointers of the recorded calls: their buffers must outlive it.
+ */
+typedef struct dlm_loop dlm_loop;
+int dlm_loop_begin(int32_t* steps_out);
+int dlm_loop_end(const int32_t* n_edits, int64_t batch, int32_t max_steps, dlm_loop** loop);
+int dlm_loop_cancel(void);
+int dlm_loop_launch(dlm_loop* loop);
+int dlm_loop_destroy(dlm_loop* loop);
 
 /* Sets the CUDA stream (a cudaStream_t) used by later calls on this thread. */
 int dlm_set_stream(void* stream);

@@ -56,6 +56,13 @@ def _load():
     for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
               "dlm_refine_step_static", "dlm_set_stream", "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
+    lib.dlm_loop_begin.argtypes = [ctypes.c_void_p]
+    lib.dlm_loop_end.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
+    lib.dlm_loop_cancel.argtypes = []
+    lib.dlm_loop_launch.argtypes = [ctypes.c_void_p]
+    lib.dlm_loop_destroy.argtypes = [ctypes.c_void_p]
+    for f in ("dlm_loop_begin", "dlm_loop_end", "dlm_loop_cancel", "dlm_loop_launch", "dlm_loop_destroy"):
+        getattr(lib, f).restype = ctypes.c_int
     lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
     lib.dlm_get_stream.restype = ctypes.c_void_p
     lib.dlm_status_string.restype = ctypes.c_char_p
@@ -198,6 +205,55 @@ def dlm_refine_step_static(logits, tokens, mask, params: RefineParams, argmax, c
     cp = params.to_c()
     _check(lib.dlm_refine_step_static(*[_ref(d) for d in ins], ctypes.byref(cp), *[_ref(d) for d in outs]))
     return argmax, conf, lse, new_tokens, new_mask, n_edits
+
+
+class RefineLoop:
+    """A recorded refine pass that the GPU repeats until no confident edit
+    remains or max_steps passes have run (one graph launch)."""
+
+    def __init__(self, handle: int, device: torch.device, steps_out: torch.Tensor):
+        self._h = handle
+        self.device = device
+        self.steps_out = steps_out
+
+    def launch(self):
+        """Runs the loop on the current stream of its device; steps_out then
+        holds the number of passes once the stream reaches that point."""
+        if not self._h:
+            raise ValueError("the loop has been destroyed")
+        torch.cuda.set_device(self.device)
+        _check(lib.dlm_set_stream(ctypes.c_void_p(torch.cuda.current_stream(self.device).cuda_stream)))
+        _check(lib.dlm_loop_launch(ctypes.c_void_p(self._h)))
+
+    def close(self):
+        if self._h:
+            _check(lib.dlm_loop_destroy(ctypes.c_void_p(self._h)))
+            self._h = None
+
+
+def dlm_loop_begin(steps_out: torch.Tensor):
+    """Starts recording one refine pass on the current (non-default) stream."""
+    if steps_out.dtype != torch.int32 or steps_out.numel() != 1:
+        raise ValueError("steps_out must be a one-element int32 CUDA tensor")
+    _prepare(steps_out)
+    _check(lib.dlm_loop_begin(ctypes.c_void_p(steps_out.data_ptr())))
+
+
+def dlm_loop_end(n_edits: torch.Tensor, max_steps: int, steps_out: torch.Tensor) -> RefineLoop:
+    """Ends the recording: the pass repeats while passes < max_steps and some
+    n_edits[b] > 0."""
+    if n_edits.dtype != torch.int32 or not n_edits.is_contiguous() or n_edits.dim() != 1:
+        lib.dlm_loop_cancel()
+        raise ValueError("n_edits must be a contiguous int32 [B] CUDA tensor")
+    h = ctypes.c_void_p()
+    _check(lib.dlm_loop_end(ctypes.c_void_p(n_edits.data_ptr() if n_edits.numel() else None), n_edits.numel(),
+                            int(max_steps), ctypes.byref(h)))
+    return RefineLoop(h.value, n_edits.device, steps_out)
+
+
+def dlm_loop_cancel():
+    """Ends an unfinished recording on this thread, keeping nothing."""
+    _check(lib.dlm_loop_cancel())
 
 
 def device_error(clear: bool = True) -> int:

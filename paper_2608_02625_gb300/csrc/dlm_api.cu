@@ -115,6 +115,10 @@ int fail(int status, const char* fmt, ...) {
   return status;
 }
 
+void clear_error() { t_last_error[0] = '\0'; }
+
+cudaStream_t current_stream() { return t_stream; }
+
 int* device_error_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;

@@ -14,6 +14,10 @@ int* device_error_word();
 
 // Records a failure message for dlm_last_error() and returns `status`.
 int fail(int status, const char* fmt, ...);
+// Clears the calling thread's failure message (at the start of every entry point).
+void clear_error();
+// The calling thread's stream (dlm_set_stream).
+cudaStream_t current_stream();
 
 struct AttnArgs {
   const void* q;

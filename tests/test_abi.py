@@ -248,3 +248,16 @@ def test_static_step_rejects_batch_above_maximum_on_the_host():
                                     r(d["ls"]), r(d["nt"]), r(d["nm"]), r(d["ne"]))
     assert st == -3
     assert b"4096" in lib.dlm_last_error()
+
+
+def test_loop_calls_rejected_on_the_host():
+    from paper_2608_02625_gb300.binding import lib
+    assert lib.dlm_set_stream(None) == 0
+    steps = ctypes.c_void_p(13 * MB)
+    assert lib.dlm_loop_begin(steps) == -6                   # legacy default stream cannot be recorded
+    assert b"stream" in lib.dlm_last_error()
+    h = ctypes.c_void_p()
+    assert lib.dlm_loop_end(ctypes.c_void_p(7 * MB), 2, 4, ctypes.byref(h)) == -6   # nothing recorded
+    assert lib.dlm_loop_cancel() == 0
+    assert lib.dlm_loop_launch(None) == -1
+    assert lib.dlm_loop_destroy(None) == 0
