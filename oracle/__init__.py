@@ -18,7 +18,9 @@ which any response position may be revised. One pass on the hot path is
   edits, Table 10 "Refine th." and Appendix C.4's confident edits);
 * ``update.refine_update``      -- commit masked positions, edit confident
   changes of filled draft tokens, remask the k least confident positions
-  (Appendix C.4, Table 11: token editing that stops when no confident edits remain).
+  (Appendix C.4, Table 11: token editing that stops when no confident edits remain);
+  optionally ranked by the probability of each position's resulting token,
+  with ``vocab.token_prob`` giving the probability of a kept token.
 
 Floating point is fp64 unless a comparison is defined in fp32 (edit threshold,
 remask order), where the fp32 values are compared exactly.
@@ -28,5 +30,5 @@ itself: brute-force loops on tiny inputs, torch fp64 library routines, closed
 forms, invariants and hand-worked update examples (tests/golden/).
 """
 from .attention import bidir_attn  # noqa: F401
-from .vocab import vocab_confidence  # noqa: F401
+from .vocab import token_prob, vocab_confidence  # noqa: F401
 from .update import refine_update, remask_count  # noqa: F401

@@ -21,6 +21,14 @@ r_b = n_b - p_b):
 The threshold compare and the remask order use the fp32 values as given
 (-0.0 and +0.0 compare equal). seq_lens is clamped to [0, L] and prompt_lens
 to [0, n_b].
+
+Variant (a second reading of step 4, when ``tok_prob`` is given): the remask
+order ranks each response position by the probability of the token it holds
+after step 2 -- conf_i when that token is the argmax (commit, edit, or a kept
+token equal to the argmax), else tok_prob_i, the softmax probability of the
+kept token (``vocab.token_prob``) -- so the least likely resulting tokens are
+remasked. The paper does not fix which of the two rankings its editing rule
+uses; the default is the first.
 """
 from __future__ import annotations
 
@@ -55,15 +63,22 @@ def remask_order(conf_vals, positions):
     return sorted(positions, key=lambda i: (conf_vals[i], i))
 
 
+def resulting_token_prob(new_tok: int, pred: int, c: float, tp: float) -> float:
+    """Probability of the token a position holds after step 2 (variant ranking)."""
+    return c if new_tok == pred else tp
+
+
 def refine_update(tokens, mask, argmax, conf, *, edit_threshold, remask_k, remask_frac,
-                  mask_id, prompt_lens, seq_lens):
-    """tokens int [B,L], mask uint8 [B,L], argmax int [B,L], conf f32 [B,L].
+                  mask_id, prompt_lens, seq_lens, tok_prob=None):
+    """tokens int [B,L], mask uint8 [B,L], argmax int [B,L], conf f32 [B,L];
+    tok_prob f32 [B,L] or None (variant ranking, see the module docstring).
 
     Returns (new_tokens int32[B,L], new_mask uint8[B,L], n_edits int32[B])."""
     tokens = np.asarray(tokens)
     mask = np.asarray(mask)
     argmax = np.asarray(argmax)
     conf32 = np.asarray(conf, dtype=np.float32)
+    tp32 = None if tok_prob is None else np.asarray(tok_prob, dtype=np.float32)
     B, L = tokens.shape
     tau = float(np.float32(edit_threshold))
     new_tok = np.array(tokens, dtype=np.int32, copy=True)
@@ -86,7 +101,12 @@ def refine_update(tokens, mask, argmax, conf, *, edit_threshold, remask_k, remas
                 new_tok[b, i] = tok[i]
             new_mask[b, i] = 0
         k = remask_count(remask_k, remask_frac, n - p)
-        for i in remask_order(c, range(p, n))[:k]:
+        rank = c
+        if tp32 is not None:
+            rank = list(c)
+            for i in range(p, n):
+                rank[i] = resulting_token_prob(int(new_tok[b, i]), pred[i], c[i], float(tp32[b, i]))
+        for i in remask_order(rank, range(p, n))[:k]:
             new_mask[b, i] = 1
             new_tok[b, i] = mask_id
         n_edits[b] = edits

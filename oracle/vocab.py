@@ -39,3 +39,26 @@ def vocab_confidence(logits, chunk_rows: int = 256):
         lse[r0:r0 + chunk_rows] = (m + np.log(S)).astype(np.float32)
         conf[r0:r0 + chunk_rows] = (1.0 / S).astype(np.float32)
     return am, conf, lse
+
+
+def token_prob(logits, tokens, lse):
+    """Softmax probability of a given token of each row: p_r = exp(x_{r,t_r} - lse_r).
+
+    logits [N, V], tokens int [N], lse [N] (the row's log-sum-exp, as given).
+    Evaluated in fp64 and rounded once to fp32; a token outside [0, V) gives 0.
+    With t_r the row's argmax this is conf_r (exp(m - lse) = 1 / S)."""
+    logits = np.asarray(logits)
+    tokens = np.asarray(tokens).reshape(-1)
+    lse = np.asarray(lse, dtype=np.float64).reshape(-1)
+    N, V = logits.shape
+    out = np.zeros(N, dtype=np.float32)
+    for r in range(N):
+        t = int(tokens[r])
+        if 0 <= t < V:
+            out[r] = np.float32(softmax_prob(np.float64(logits[r, t]), lse[r]))
+    return out
+
+
+def softmax_prob(x_t: float, lse: float) -> float:
+    """exp(x_t - lse): one entry of softmax(x) given the row's log-sum-exp."""
+    return float(np.exp(x_t - lse))

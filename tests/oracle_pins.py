@@ -210,8 +210,43 @@ def pin_vocab_torch():
     assert np.all(np.abs(conf.astype(np.float64) - ref_conf) <= 1e-7 * ref_conf)
 
 
+def pin_token_prob_closed_forms():
+    """Uniform row: 1/V for every token; two-valued row in closed form; a token
+    outside [0, V) gives 0; the argmax's probability is the confidence."""
+    V = 300
+    x = np.full((3, V), 1.25)
+    x[1, 40] = 3.0
+    lse = np.array([1.25 + math.log(V), math.log(math.exp(3.0) + (V - 1) * math.exp(1.25)), 0.0])
+    p = oracle.token_prob(x, np.array([7, 40, V]), lse)
+    assert abs(float(p[0]) - 1.0 / V) <= 1e-7 / V
+    c = math.exp(3.0) / (math.exp(3.0) + (V - 1) * math.exp(1.25))
+    assert abs(float(p[1]) - c) <= 1e-7 * c
+    assert p[2] == 0.0
+    rng = np.random.default_rng(23)
+    y = rng.standard_normal((9, 2000)) * 3.0
+    am, conf, lse32 = oracle.vocab_confidence(y)
+    pa = oracle.token_prob(y, am, lse32)
+    assert np.all(np.abs(pa.astype(np.float64) - conf) <= 1e-5 * conf)
+
+
+def pin_token_prob_torch():
+    """Against torch fp64 log_softmax + gather, and the probabilities of all
+    tokens of a row summing to 1."""
+    rng = np.random.default_rng(24)
+    x = rng.standard_normal((17, 3000)) * 2.5
+    tok = rng.integers(0, 3000, 17)
+    t = torch.from_numpy(x)
+    lse = torch.logsumexp(t, dim=1).numpy()
+    p = oracle.token_prob(x, tok, lse)
+    ref = torch.exp(torch.log_softmax(t, dim=1).gather(1, torch.from_numpy(tok)[:, None])[:, 0]).numpy()
+    assert np.all(np.abs(p.astype(np.float64) - ref) <= 1e-6 * ref + 1e-30)
+    row = np.repeat(x[:1], 3000, axis=0)
+    tot = oracle.token_prob(row, np.arange(3000), np.full(3000, lse[0])).astype(np.float64).sum()
+    assert abs(tot - 1.0) <= 1e-5
+
+
 VOCAB_PINS = [pin_vocab_uniform_row, pin_vocab_single_finite, pin_vocab_two_valued_closed_form,
-              pin_vocab_ties_lowest_index, pin_vocab_torch]
+              pin_vocab_ties_lowest_index, pin_vocab_torch, pin_token_prob_closed_forms, pin_token_prob_torch]
 
 
 # ---------------------------------------------------------------- update
@@ -226,10 +261,11 @@ def run_case(c):
     m = np.array([c["mask"]], dtype=np.uint8)
     am = np.array([c["argmax"]], dtype=np.int32)
     cf = np.array([c["conf"]], dtype=np.float32)
+    tp = np.array([c["tok_prob"]], dtype=np.float32) if "tok_prob" in c else None
     return oracle.refine_update(tok, m, am, cf, edit_threshold=c["edit_threshold"],
                                 remask_k=c["remask_k"], remask_frac=c["remask_frac"],
                                 mask_id=c["mask_id"], prompt_lens=[c["prompt_len"]],
-                                seq_lens=[c["seq_len"]])
+                                seq_lens=[c["seq_len"]], tok_prob=tp)
 
 
 def pin_update_golden():
@@ -329,7 +365,43 @@ def pin_update_remask_fraction():
     assert oupd.remask_count(5, 0.9, 3) == 3
 
 
+def pin_update_result_ranking():
+    """Ranking by the resulting token's probability: with tok_prob = conf it is
+    the default ranking; otherwise position i is remasked iff fewer than k
+    response positions j have (key_j, j) < (key_i, i), key = conf where the
+    position ends with its argmax and tok_prob elsewhere (O(r^2) rank count);
+    steps 1-2 and the edit count do not depend on the ranking."""
+    rng = np.random.default_rng(33)
+    for trial in range(20):
+        case = random_update_case(rng, B=3, L=30, ties=trial % 2 == 0)
+        k = int(rng.integers(0, 20))
+        args = dict(edit_threshold=0.5, remask_k=k, remask_frac=0.0, mask_id=case["V"],
+                    prompt_lens=case["prompt_lens"], seq_lens=case["seq_lens"])
+        base = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"], **args)
+        same = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"],
+                                    tok_prob=case["conf"], **args)
+        for x, y in zip(base, same):
+            assert np.array_equal(x, y)
+        tp = rng.choice(np.array([0.0, 0.1, 0.5], dtype=np.float32), (3, 30)) if trial % 2 == 0 else \
+            rng.random((3, 30)).astype(np.float32)
+        nt, nm, ne = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"],
+                                          tok_prob=tp, **args)
+        assert np.array_equal(ne, base[2])
+        unmasked = (nm == 0) & (base[1] == 0)
+        assert np.array_equal(nt[unmasked], base[0][unmasked])
+        am, cf = case["argmax"], case["conf"]
+        for b in range(3):
+            p, n = int(case["prompt_lens"][b]), int(case["seq_lens"][b])
+            after = [int(am[b, i]) if case["mask"][b, i] or (am[b, i] != case["tokens"][b, i] and
+                                                              cf[b, i] >= np.float32(0.5))
+                     else int(case["tokens"][b, i]) for i in range(30)]
+            key = [float(cf[b, i]) if after[i] == int(am[b, i]) else float(tp[b, i]) for i in range(30)]
+            for i in range(p, n):
+                rank = sum(1 for j in range(p, n) if (key[j] < key[i]) or (key[j] == key[i] and j < i))
+                assert (nm[b, i] == 1) == (rank < k)
+
+
 UPDATE_PINS = [pin_update_golden, pin_update_invariants, pin_update_rank_count,
-               pin_update_remask_fraction]
+               pin_update_remask_fraction, pin_update_result_ranking]
 
 ALL_PINS = ATTN_PINS + VOCAB_PINS + UPDATE_PINS

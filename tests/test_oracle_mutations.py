@@ -3,7 +3,9 @@
 Every mutation below is a plausible slip in writing the method down: a causal
 mask, a wrong softmax scale, interleaved instead of contiguous GQA groups, the
 last instead of the first maximum, a strict threshold, ties broken towards the
-higher index, a rounded-up remask count. If a pin suite let one through, the
+higher index, a rounded-up remask count, a resulting-token ranking that
+ignores which positions end with their argmax, a sign slip in a token's
+probability. If a pin suite let one through, the
 oracle could carry that slip undetected."""
 import math
 
@@ -24,6 +26,8 @@ MUTATIONS = {
     "strict_threshold": (oupd, "is_edit", lambda p, t, c, tau: p != t and c > tau, P.UPDATE_PINS),
     "ties_high_index": (oupd, "remask_order",
                         lambda cv, pos: sorted(pos, key=lambda i: (cv[i], -i)), P.UPDATE_PINS),
+    "result_rank_ignores_argmax": (oupd, "resulting_token_prob", lambda nt, pred, c, tp: tp, P.UPDATE_PINS),
+    "token_prob_sign": (ovoc, "softmax_prob", lambda x, lse: float(np.exp(lse - x)), P.VOCAB_PINS),
     "ceil_remask_count": (oupd, "remask_count",
                           lambda k, f, r: max(0, min(k if k >= 0 else
                                                      math.ceil(float(np.float32(f)) * r), r)),
