@@ -348,6 +348,36 @@ def measure_loop(args, w, Bn, q, k, v, out, logits, tok0, msk0, params, seqlen, 
                     "graph: CUDA events around one launch; host-driven: wall clock, one n_edits read-back per pass"}
 
 
+def measure_ranked(Bn, w, logits, tok, msk, am, cf, ls, params, stream, reps=20):
+    """Remask ranking by the resulting token's probability: dlm_token_prob of
+    the current tokens plus dlm_refine_update_ranked, timed with CUDA events
+    (mean per launch) on the bench workload's resident inputs."""
+    import torch
+    d = tok.device
+    pr = torch.empty(w.N, dtype=torch.float32, device=d)
+    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    am2, cf2, pr2 = am.view(w.B, w.L), cf.view(w.B, w.L), pr.view(w.B, w.L)
+    for _ in range(3):
+        Bn.dlm_token_prob(logits, tok.view(-1), ls, pr)
+        Bn.dlm_refine_update_ranked(tok, msk, am2, cf2, pr2, params, nt, nm, ne)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    t_tp = t_up = 0.0
+    for _ in range(reps):
+        ev[0].record(stream)
+        Bn.dlm_token_prob(logits, tok.view(-1), ls, pr)
+        ev[1].record(stream)
+        Bn.dlm_refine_update_ranked(tok, msk, am2, cf2, pr2, params, nt, nm, ne)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        t_tp += ev[0].elapsed_time(ev[1])
+        t_up += ev[1].elapsed_time(ev[2])
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the ranked-update measurement")
+    return {"token_prob_ms": t_tp / reps, "update_ranked_ms": t_up / reps,
+            "note": "remask ranking by the resulting token's probability (variant reading); not in the step"}
+
+
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -488,6 +518,7 @@ def run_ours(args, rank, world):
 
     # ---- multi-pass refinement: the recorded pass repeated by one graph launch
     # (device-side early stop) against the same passes driven from the host
+    ranked_info = measure_ranked(Bn, w, logits, tok, msk, am, cf, ls, params, stream)
     loop_info = None
     if args.loop_steps > 0:
         loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
@@ -537,6 +568,7 @@ def run_ours(args, rank, world):
         "path": args.path,
         "e2e": e2e,
         "loop": loop_info,
+        "ranked_variant": ranked_info,
     }
     if timer is not None:
         res["cpu_baseline"] = timer.run()

@@ -164,6 +164,34 @@ int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dl
                       dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits);
 
 /*
+ * Probability of a given token of each row under the row's softmax:
+ *   prob[r] = exp(logits[r, tokens[r]] - lse[r]),   0 if tokens[r] is outside [0, V).
+ * With lse from dlm_vocab_confidence and tokens[r] the current token of a
+ * position, this is the probability the refiner assigns to keeping it; it
+ * feeds the remask ranking of dlm_refine_update_ranked.
+ *   logits  as for dlm_vocab_confidence;  tokens N I32, lse N F32, prob N F32
+ *   (any rank with N elements, contiguous). fp32: one gathered logit per row.
+ */
+int dlm_token_prob(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* lse,
+                   dlm_tensor* prob);
+
+/*
+ * dlm_refine_update with the remask ranking of a second reading of the paper's
+ * editing rule (Appendix C.4 / Table 11 do not fix which probability ranks the
+ * positions to remask): step 4 orders the response positions by the
+ * probability of the token each holds after step 2 -- conf[i] where that
+ * token is the argmax (commit, edit, or a kept token equal to the argmax),
+ * tok_prob[i] (the kept token's probability, dlm_token_prob) elsewhere --
+ * ascending, index ascending. Steps 1-3 and 5 are those of dlm_refine_update.
+ *   tok_prob  [B, L] F32 (innermost contiguous); the other arguments as for
+ *             dlm_refine_update. Bit-exact (exact fp32 compares only).
+ */
+int dlm_refine_update_ranked(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
+                             const dlm_tensor* conf, const dlm_tensor* tok_prob,
+                             const dlm_refine_params* params, dlm_tensor* new_tokens,
+                             dlm_tensor* new_mask, dlm_tensor* n_edits);
+
+/*
  * Steps A2 and A3 fused in one launch (the per-position reduction of the
  * confidences of Table 10 / Appendix C.4 feeding the update of Sec. 4.2).
  * Computes exactly what dlm_vocab_confidence(logits, argmax, conf, lse)

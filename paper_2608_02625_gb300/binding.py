@@ -50,11 +50,14 @@ def _load():
     lib.dlm_refine_update.argtypes = [P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
     lib.dlm_refine_step.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P,
                                     ctypes.c_void_p, ctypes.c_size_t]
+    lib.dlm_token_prob.argtypes = [P, P, P, P]
+    lib.dlm_refine_update_ranked.argtypes = [P, P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
     lib.dlm_refine_step_static.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P]
     lib.dlm_refine_step_workspace_bytes.argtypes = [ctypes.c_int64]
     lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
     for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
-              "dlm_refine_step_static", "dlm_set_stream", "dlm_version", "dlm_get_device_error"):
+              "dlm_refine_step_static", "dlm_token_prob", "dlm_refine_update_ranked", "dlm_set_stream",
+              "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
     lib.dlm_loop_begin.argtypes = [ctypes.c_void_p]
     lib.dlm_loop_end.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
@@ -166,6 +169,26 @@ def dlm_refine_update(tokens, mask, argmax, conf, params: RefineParams, new_toke
     outs = [describe(t) for t in (new_tokens, new_mask, n_edits)]
     cp = params.to_c()
     _check(lib.dlm_refine_update(*[_ref(d) for d in ds], ctypes.byref(cp), *[_ref(d) for d in outs]))
+    return new_tokens, new_mask, n_edits
+
+
+def dlm_token_prob(logits, tokens, lse, prob):
+    """prob[r] = exp(logits[r, tokens[r]] - lse[r]) (0 for a token outside [0, V))."""
+    _prepare(logits, tokens, lse, prob)
+    ds = [describe(t) for t in (logits, tokens, lse, prob)]
+    _check(lib.dlm_token_prob(*[_ref(d) for d in ds]))
+    return prob
+
+
+def dlm_refine_update_ranked(tokens, mask, argmax, conf, tok_prob, params: RefineParams, new_tokens, new_mask,
+                             n_edits):
+    """dlm_refine_update remasking by the probability of each position's resulting token."""
+    _prepare(tokens, mask, argmax, conf, tok_prob, new_tokens, new_mask, n_edits, params.prompt_lens,
+             params.seq_lens)
+    ds = [describe(t) for t in (tokens, mask, argmax, conf, tok_prob)]
+    outs = [describe(t) for t in (new_tokens, new_mask, n_edits)]
+    cp = params.to_c()
+    _check(lib.dlm_refine_update_ranked(*[_ref(d) for d in ds], ctypes.byref(cp), *[_ref(d) for d in outs]))
     return new_tokens, new_mask, n_edits
 
 

@@ -255,15 +255,12 @@ int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v
 
 namespace {
 
-// Validates the arguments of the vocabulary reduction and fills *a.
-int prepare_vocab(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
-                  dlm::VocabArgs* a) {
+// Validates a logits descriptor ([N, V] or [B, L, V], evenly strided rows)
+// and fills the logits fields of *a.
+int prepare_logits(const dlm_tensor* logits, dlm::VocabArgs* a) {
   using dlm::fail;
   int st;
   if ((st = check_tensor(logits, "logits", kMaskBF16F32, 2, 3))) return st;
-  if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 1, 3))) return st;
-  if ((st = check_tensor(conf, "conf", 1 << DLM_F32, 1, 3))) return st;
-  if ((st = check_tensor(lse, "lse", 1 << DLM_F32, 1, 3))) return st;
   const int nd = logits->ndim;
   const int64_t V = logits->shape[nd - 1];
   int64_t N = 1;
@@ -274,6 +271,24 @@ int prepare_vocab(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf
     return fail(DLM_ERR_STRIDE, "logits rows must be evenly strided ([B, L, V] with stride[0] = L * stride[1])");
   if (N > 0 && V < 1) return fail(DLM_ERR_SHAPE, "V must be >= 1");
   if (N > 1 && row_stride < V) return fail(DLM_ERR_STRIDE, "logits rows overlap");
+  a->logits = logits->data;
+  a->is_bf16 = logits->dtype == DLM_BF16;
+  a->N = N;
+  a->V = V;
+  a->row_stride = N > 1 ? row_stride : V;
+  return DLM_OK;
+}
+
+// Validates the arguments of the vocabulary reduction and fills *a.
+int prepare_vocab(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf, dlm_tensor* lse,
+                  dlm::VocabArgs* a) {
+  using dlm::fail;
+  int st;
+  if ((st = prepare_logits(logits, a))) return st;
+  if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 1, 3))) return st;
+  if ((st = check_tensor(conf, "conf", 1 << DLM_F32, 1, 3))) return st;
+  if ((st = check_tensor(lse, "lse", 1 << DLM_F32, 1, 3))) return st;
+  const int64_t N = a->N;
   const dlm_tensor* outs[3] = {argmax, conf, lse};
   for (const dlm_tensor* t : outs) {
     if (numel(t) != N) return fail(DLM_ERR_SHAPE, "argmax, conf and lse must have one entry per logits row");
@@ -282,11 +297,6 @@ int prepare_vocab(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tensor* conf
   }
   if (overlaps(argmax, conf) || overlaps(argmax, lse) || overlaps(conf, lse))
     return fail(DLM_ERR_ARG, "outputs overlap each other");
-  a->logits = logits->data;
-  a->is_bf16 = logits->dtype == DLM_BF16;
-  a->N = N;
-  a->V = V;
-  a->row_stride = N > 1 ? row_stride : V;
   a->argmax = static_cast<int32_t*>(argmax->data);
   a->conf = static_cast<float*>(conf->data);
   a->lse = static_cast<float*>(lse->data);
@@ -355,6 +365,8 @@ int prepare_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_t
   a->mask_id = params->mask_id;
   a->prompt_lens = params->prompt_lens;
   a->seq_lens = params->seq_lens;
+  a->tok_prob = nullptr;
+  a->s_tok_prob = 0;
   return DLM_OK;
 }
 
@@ -406,6 +418,49 @@ int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dl
   int st = prepare_update(tokens, mask, argmax, conf, params, new_tokens, new_mask, n_edits, &a);
   if (st != DLM_OK || a.B == 0) return st;
   if ((st = require_error_word())) return st;
+  return dlm::launch_refine_update(a, t_stream);
+}
+
+int dlm_token_prob(const dlm_tensor* logits, const dlm_tensor* tokens, const dlm_tensor* lse, dlm_tensor* prob) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  int st;
+  dlm::VocabArgs a = {};
+  if ((st = prepare_logits(logits, &a))) return st;
+  if ((st = check_tensor(tokens, "tokens", 1 << DLM_I32, 1, 3))) return st;
+  if ((st = check_tensor(lse, "lse", 1 << DLM_F32, 1, 3))) return st;
+  if ((st = check_tensor(prob, "prob", 1 << DLM_F32, 1, 3))) return st;
+  const int64_t N = a.N;
+  if (numel(tokens) != N || numel(lse) != N || numel(prob) != N)
+    return fail(DLM_ERR_SHAPE, "tokens, lse and prob must have one entry per logits row");
+  if (!is_dense(tokens) || !is_dense(lse) || !is_dense(prob))
+    return fail(DLM_ERR_STRIDE, "tokens, lse and prob must be contiguous");
+  if (overlaps(prob, logits) || overlaps(prob, tokens) || overlaps(prob, lse))
+    return fail(DLM_ERR_ARG, "prob overlaps an input");
+  if (N == 0) return DLM_OK;
+  if ((st = require_error_word())) return st;
+  return dlm::launch_token_prob(a, static_cast<const int32_t*>(tokens->data), static_cast<const float*>(lse->data),
+                                static_cast<float*>(prob->data), t_stream);
+}
+
+int dlm_refine_update_ranked(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
+                             const dlm_tensor* conf, const dlm_tensor* tok_prob, const dlm_refine_params* params,
+                             dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  dlm::UpdateArgs a;
+  int st = prepare_update(tokens, mask, argmax, conf, params, new_tokens, new_mask, n_edits, &a);
+  if (st != DLM_OK) return st;
+  if ((st = check_tensor(tok_prob, "tok_prob", 1 << DLM_F32, 2, 2))) return st;
+  if (tok_prob->shape[0] != a.B || tok_prob->shape[1] != a.L)
+    return fail(DLM_ERR_SHAPE, "tok_prob must be [B, L]");
+  const dlm_tensor* outs[3] = {new_tokens, new_mask, n_edits};
+  for (const dlm_tensor* o : outs)
+    if (overlaps(o, tok_prob)) return fail(DLM_ERR_ARG, "an output overlaps tok_prob");
+  if (a.B == 0) return DLM_OK;
+  if ((st = require_error_word())) return st;
+  a.tok_prob = static_cast<const float*>(tok_prob->data);
+  a.s_tok_prob = tok_prob->stride[0];
   return dlm::launch_refine_update(a, t_stream);
 }
 

@@ -60,9 +60,17 @@ struct UpdateArgs {
   int32_t mask_id;
   const int32_t* prompt_lens;
   const int32_t* seq_lens;
+  // Remask ranking by the resulting token's probability when non-null: the
+  // probability of each position's current token, [B, L] with sequence stride s_tok_prob.
+  const float* tok_prob;
+  int64_t s_tok_prob;
 };
 
 int launch_refine_update(const UpdateArgs& a, cudaStream_t stream);
+
+// prob[r] = exp(logits[r, tokens[r]] - lse[r]) (0 for a token outside [0, V)).
+int launch_token_prob(const VocabArgs& a, const int32_t* tokens, const float* lse, float* prob,
+                      cudaStream_t stream);
 
 // Fused vocabulary reduction + update (rows of sequence b are b * L .. b * L + L - 1;
 // u.argmax / u.conf alias a.argmax / a.conf). counters: int32[B], zero on entry.

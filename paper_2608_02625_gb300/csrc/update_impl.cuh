@@ -8,7 +8,10 @@
 //           differs and whose conf >= tau; count edits (block reduction);
 //   pass 2  radix select over the response keys: the k_b-th smallest of
 //           key(conf) (an order-preserving map of the fp32 bits, -0 -> +0),
-//           4 passes of 8 bits with warp-aggregated shared-memory histograms;
+//           4 passes of 8 bits with warp-aggregated shared-memory histograms
+//           (with a.tok_prob, key of the probability of the token each
+//           position holds after pass 1: conf where that is the argmax, the
+//           given probability of the kept token elsewhere);
 //   pass 3  remask keys below the k-th key, and the lowest-index positions
 //           whose key equals it (an ordered block scan), up to k_b in total.
 // Integer work and exact fp32 compares only: results are bit-exact.
@@ -103,6 +106,12 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
   const float* cf = a.conf + b * a.s_conf;
   int32_t* ntok = a.new_tokens + b * a.s_new_tokens;
   uint8_t* nmsk = a.new_mask + b * a.s_new_mask;
+  const float* tp = a.tok_prob ? a.tok_prob + b * a.s_tok_prob : nullptr;
+  // Ranking value of response position i once pass 1 has written new_tokens.
+  auto rank_value = [&](int i) -> float {
+    if (tp && ntok[i] != load_pred<kFresh>(am + i)) return tp[i];
+    return load_pred<kFresh>(cf + i);
+  };
 
   // ---- pass 1: copy / commit / edit (read and write of position i by one
   // thread, so new_* may alias tokens/mask)
@@ -158,7 +167,7 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
       bool active = false;
       uint32_t digit = 0;
       if (i < n) {
-        const float c = load_pred<kFresh>(cf + i);
+        const float c = rank_value(i);
         if (shift == 24 && is_nan_bits(__float_as_uint(c))) saw_nan = true;
         uint32_t key = conf_key(c);
         if ((key & pmask) == prefix) {
@@ -210,7 +219,7 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
   int taken = 0;
   for (int base = p; base < n; base += kThreads) {
     int i = base + tid;
-    uint32_t key = i < n ? conf_key(load_pred<kFresh>(cf + i)) : 0xFFFFFFFFu;
+    uint32_t key = i < n ? conf_key(rank_value(i)) : 0xFFFFFFFFu;
     bool eq = i < n && key == kth;
     int total;
     int incl = block_inclusive_scan<kThreads>(eq ? 1 : 0, sh.warp_sums, &total);

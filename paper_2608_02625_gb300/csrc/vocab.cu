@@ -286,6 +286,23 @@ __global__ void __launch_bounds__(kThreads, 4) vocab_cluster_kernel(VocabArgs a)
   cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
 }
 
+// Probability of a given token of each row: one gathered logit per row.
+template <bool BF16>
+__global__ void __launch_bounds__(256) token_prob_kernel(VocabArgs a, const int32_t* tokens, const float* lse,
+                                                         float* prob) {
+  const int64_t r = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (r >= a.N) return;
+  const int32_t t = tokens[r];
+  float p = 0.f;
+  if (t >= 0 && t < a.V) {
+    const int64_t off = r * a.row_stride + t;
+    const float x = BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(a.logits)[off])
+                         : static_cast<const float*>(a.logits)[off];
+    p = expf(x - lse[r]);
+  }
+  prob[r] = p;
+}
+
 template <bool BF16, bool VEC>
 int launch_typed(const VocabArgs& a, cudaStream_t stream) {
   int dev = 0, sms = 0;
@@ -330,6 +347,17 @@ int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream) {
   const bool vec = (reinterpret_cast<uintptr_t>(a.logits) % 16 == 0) && ((a.row_stride * esz) % 16 == 0);
   if (a.is_bf16) return vec ? launch_typed<true, true>(a, stream) : launch_typed<true, false>(a, stream);
   return vec ? launch_typed<false, true>(a, stream) : launch_typed<false, false>(a, stream);
+}
+
+int launch_token_prob(const VocabArgs& a, const int32_t* tokens, const float* lse, float* prob,
+                      cudaStream_t stream) {
+  if (a.N == 0) return DLM_OK;
+  const unsigned grid = static_cast<unsigned>((a.N + 255) / 256);
+  if (a.is_bf16) token_prob_kernel<true><<<grid, 256, 0, stream>>>(a, tokens, lse, prob);
+  else token_prob_kernel<false><<<grid, 256, 0, stream>>>(a, tokens, lse, prob);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "token_prob launch: %s", cudaGetErrorString(e));
+  return DLM_OK;
 }
 
 int launch_vocab_step(const VocabArgs& a, const UpdateArgs& u, int* counters, cudaStream_t stream) {

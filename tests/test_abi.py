@@ -261,3 +261,43 @@ def test_loop_calls_rejected_on_the_host():
     assert lib.dlm_loop_cancel() == 0
     assert lib.dlm_loop_launch(None) == -1
     assert lib.dlm_loop_destroy(None) == 0
+
+
+@pytest.mark.parametrize("case,status", [
+    ("ok_shape_mismatch", -3), ("tokens_f32", -2), ("strided_prob", -4), ("prob_overlaps_lse", -6), ("null_lse", -1),
+])
+def test_token_prob_rejects(case, status):
+    from paper_2608_02625_gb300.binding import lib
+    lg, tk, ls, pr = T(BF16, [4, 1000], 1 * MB), T(I32, [4], 2 * MB), T(F32, [4], 3 * MB), T(F32, [4], 4 * MB)
+    if case == "ok_shape_mismatch":
+        tk = T(I32, [5], 2 * MB)
+    elif case == "tokens_f32":
+        tk = T(F32, [4], 2 * MB)
+    elif case == "strided_prob":
+        pr = T(F32, [4], 4 * MB, strides=[2])
+    elif case == "prob_overlaps_lse":
+        pr = T(F32, [4], 3 * MB + 4)
+    elif case == "null_lse":
+        ls = None
+    r = lambda x: ctypes.byref(x) if x is not None else None
+    assert lib.dlm_token_prob(r(lg), r(tk), r(ls), r(pr)) == status
+
+
+@pytest.mark.parametrize("case,status", [("tok_prob_shape", -3), ("tok_prob_dtype", -2), ("out_overlaps_tok_prob", -6),
+                                         ("null_tok_prob", -1)])
+def test_update_ranked_rejects(case, status):
+    from paper_2608_02625_gb300.binding import lib
+    d = dict(tok=T(I32, [2, 8], 1 * MB), msk=T(U8, [2, 8], 2 * MB), am=T(I32, [2, 8], 3 * MB),
+             cf=T(F32, [2, 8], 4 * MB), tp=T(F32, [2, 8], 10 * MB), nt=T(I32, [2, 8], 5 * MB),
+             nm=T(U8, [2, 8], 6 * MB), ne=T(I32, [2], 7 * MB))
+    if case == "tok_prob_shape":
+        d["tp"] = T(F32, [2, 9], 10 * MB)
+    elif case == "tok_prob_dtype":
+        d["tp"] = T(I32, [2, 8], 10 * MB)
+    elif case == "out_overlaps_tok_prob":
+        d["nt"] = T(I32, [2, 8], 10 * MB)
+    elif case == "null_tok_prob":
+        d["tp"] = None
+    r = lambda x: ctypes.byref(x) if x is not None else None
+    assert lib.dlm_refine_update_ranked(r(d["tok"]), r(d["msk"]), r(d["am"]), r(d["cf"]), r(d["tp"]), r(P()),
+                                        r(d["nt"]), r(d["nm"]), r(d["ne"])) == status

@@ -37,8 +37,9 @@ def assert_same(gpu, ref, where=""):
         assert np.array_equal(g, r), f"{where}: {name} differs at {np.argwhere(g != r)[:8].tolist()}"
 
 
-@pytest.mark.parametrize("case", P.golden_cases(), ids=lambda c: c["name"])
+@pytest.mark.parametrize("case", [c for c in P.golden_cases() if "tok_prob" not in c], ids=lambda c: c["name"])
 def test_golden_cases(case):
+    """The default-ranking cases (cases with a tok_prob are for dlm_refine_update_ranked)."""
     tok = np.array([case["tokens"]]); msk = np.array([case["mask"]])
     am = np.array([case["argmax"]]); cf = np.array([case["conf"]], dtype=np.float32)
     gpu = run_gpu(tok, msk, am, cf, tau=case["edit_threshold"], k=case["remask_k"], frac=case["remask_frac"],
