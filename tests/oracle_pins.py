@@ -155,9 +155,96 @@ def pin_attn_padding_and_empty():
     assert np.all(np.isfinite(got))
 
 
+def key_ranges(i, n, p, block, mode):
+    """The keys query i may use, written as index ranges (an independent
+    statement of the block variants): block-causal [0, end_i), block-local
+    [0, p) + [start_i, end_i), with start_i / end_i the bounds of i's block;
+    prompt queries [0, p)."""
+    if mode == 0:
+        return [(0, n)]
+    if i < p:
+        return [(0, p)]
+    start = p + ((i - p) // block) * block
+    end = min(n, start + block)
+    return [(0, end)] if mode == 1 else [(0, p), (start, end)]
+
+
+def brute_masked(q, k, v, seq_lens, prompt_lens, block, mode):
+    B, L, Hq, D = q.shape
+    grp = Hq // k.shape[2]
+    out = np.zeros((B, L, Hq, D))
+    for b in range(B):
+        n, p = int(seq_lens[b]), int(prompt_lens[b])
+        for h in range(Hq):
+            g = h // grp
+            for i in range(n):
+                js = [j for lo, hi in key_ranges(i, n, p, block, mode) for j in range(lo, hi)]
+                s = [float(np.dot(q[b, i, h], k[b, j, g])) / math.sqrt(D) for j in js]
+                mx = max(s)
+                w = [math.exp(x - mx) for x in s]
+                out[b, i, h] = sum(wj * v[b, j, g] for wj, j in zip(w, js)) / sum(w)
+    return out
+
+
+def pin_attn_masks_brute_force():
+    """Both block variants against loops over the key ranges, several block
+    sizes, prompts and lengths (including blocks cut by n)."""
+    rng = np.random.default_rng(18)
+    q, k, v = _rand_qkv(rng, 3, 13, 2, 1, 4)
+    sl, pl = np.array([13, 11, 5]), np.array([3, 0, 5])
+    for mode in (1, 2):
+        for block in (1, 2, 4, 20):
+            got = oracle.bidir_attn(q, k, v, sl, mask_mode=mode, block=block, prompt_lens=pl)
+            ref = brute_masked(q, k, v, sl, pl, block, mode)
+            assert np.abs(got - ref).max() < 1e-12, (mode, block)
+
+
+def pin_attn_masks_torch_sdpa():
+    """torch fp64 scaled_dot_product_attention with a boolean mask built from
+    the key ranges."""
+    rng = np.random.default_rng(19)
+    B, L, Hq, Hkv, D = 1, 40, 4, 2, 8
+    q, k, v = _rand_qkv(rng, B, L, Hq, Hkv, D)
+    n, p = 37, 6
+    for mode, block in ((1, 8), (2, 8), (1, 5)):
+        got = oracle.bidir_attn(q, k, v, [n], mask_mode=mode, block=block, prompt_lens=[p])
+        m = torch.zeros(n, n, dtype=torch.bool)
+        for i in range(n):
+            for lo, hi in key_ranges(i, n, p, block, mode):
+                m[i, lo:hi] = True
+        tq = torch.from_numpy(q[0, :n]).permute(1, 0, 2)
+        tk = torch.from_numpy(k[0, :n]).permute(1, 0, 2).repeat_interleave(Hq // Hkv, 0)
+        tv = torch.from_numpy(v[0, :n]).permute(1, 0, 2).repeat_interleave(Hq // Hkv, 0)
+        ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, attn_mask=m)
+        assert np.abs(got[0, :n] - ref.permute(1, 0, 2).numpy()).max() < 1e-12
+
+
+def pin_attn_masks_properties():
+    """Block-causal with one block covering the response is the full attention
+    for response queries; block-local with the response as one block is the
+    same; changing keys/values of a later block leaves block-causal outputs of
+    earlier blocks unchanged; prompt queries see only the prompt."""
+    rng = np.random.default_rng(20)
+    q, k, v = _rand_qkv(rng, 1, 16, 2, 2, 4)
+    n, p = 16, 4
+    full = oracle.bidir_attn(q, k, v, [n])
+    for mode in (1, 2):
+        one = oracle.bidir_attn(q, k, v, [n], mask_mode=mode, block=n - p, prompt_lens=[p])
+        assert np.abs(one[0, p:] - full[0, p:]).max() < 1e-12
+        prompt_only = oracle.bidir_attn(q, k, v, [p])
+        assert np.abs(one[0, :p] - prompt_only[0, :p]).max() < 1e-12
+    a = oracle.bidir_attn(q, k, v, [n], mask_mode=1, block=4, prompt_lens=[p])
+    k2, v2 = k.copy(), v.copy()
+    k2[0, 12:] += 3.0
+    v2[0, 12:] -= 2.0
+    b = oracle.bidir_attn(q, k2, v2, [n], mask_mode=1, block=4, prompt_lens=[p])
+    assert np.abs(a[0, :12] - b[0, :12]).max() < 1e-12 and np.abs(a[0, 12:] - b[0, 12:]).max() > 1e-3
+
+
 ATTN_PINS = [pin_attn_brute_force, pin_attn_torch_sdpa, pin_attn_identical_keys_mean,
              pin_attn_dominant_key, pin_attn_single_position, pin_attn_two_key_closed_form,
-             pin_attn_permutation_invariance, pin_attn_gqa_grouping, pin_attn_padding_and_empty]
+             pin_attn_permutation_invariance, pin_attn_gqa_grouping, pin_attn_padding_and_empty,
+             pin_attn_masks_brute_force, pin_attn_masks_torch_sdpa, pin_attn_masks_properties]
 
 
 # ---------------------------------------------------------------- vocab

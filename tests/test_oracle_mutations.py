@@ -3,7 +3,8 @@
 Every mutation below is a plausible slip in writing the method down: a causal
 mask, a wrong softmax scale, interleaved instead of contiguous GQA groups, the
 last instead of the first maximum, a strict threshold, ties broken towards the
-higher index, a rounded-up remask count, a resulting-token ranking that
+higher index, a rounded-up remask count, a block-causal mask that drops the
+query's own block, a block-local mask without the prompt, a resulting-token ranking that
 ignores which positions end with their argmax, a sign slip in a token's
 probability. If a pin suite let one through, the
 oracle could carry that slip undetected."""
@@ -18,7 +19,18 @@ from oracle import update as oupd
 from oracle import vocab as ovoc
 
 MUTATIONS = {
-    "causal_mask": (oatt, "key_mask", lambda n: np.tril(np.ones((n, n), dtype=bool)), P.ATTN_PINS),
+    "causal_mask": (oatt, "key_mask", lambda n, p=0, block=1, mode=0: np.tril(np.ones((n, n), dtype=bool)),
+                    P.ATTN_PINS),
+    "block_causal_strict": (oatt, "key_allowed",
+                            lambda i, j, p, b, mode: True if mode == 0 else (
+                                j < p or (oatt.block_index(j, p, b) < oatt.block_index(i, p, b) if mode == 1
+                                          else oatt.block_index(j, p, b) == oatt.block_index(i, p, b))),
+                            P.ATTN_PINS),
+    "local_without_prompt": (oatt, "key_allowed",
+                             lambda i, j, p, b, mode: True if mode == 0 else (
+                                 (j < p or oatt.block_index(j, p, b) <= oatt.block_index(i, p, b)) if mode == 1
+                                 else oatt.block_index(j, p, b) == oatt.block_index(i, p, b)),
+                             P.ATTN_PINS),
     "scale_1_over_D": (oatt, "score_scale", lambda D: 1.0 / D, P.ATTN_PINS),
     "interleaved_gqa": (oatt, "kv_head", lambda h, Hq, Hkv: h % Hkv, P.ATTN_PINS),
     "last_argmax": (ovoc, "first_argmax",
