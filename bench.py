@@ -348,36 +348,6 @@ def measure_loop(args, w, Bn, q, k, v, out, logits, tok0, msk0, params, seqlen, 
                     "graph: CUDA events around one launch; host-driven: wall clock, one n_edits read-back per pass"}
 
 
-def measure_ranked(Bn, w, logits, tok, msk, am, cf, ls, params, stream, reps=20):
-    """Remask ranking by the resulting token's probability: dlm_token_prob of
-    the current tokens plus dlm_refine_update_ranked, timed with CUDA events
-    (mean per launch) on the bench workload's resident inputs."""
-    import torch
-    d = tok.device
-    pr = torch.empty(w.N, dtype=torch.float32, device=d)
-    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
-    ne = torch.empty(w.B, dtype=torch.int32, device=d)
-    am2, cf2, pr2 = am.view(w.B, w.L), cf.view(w.B, w.L), pr.view(w.B, w.L)
-    for _ in range(3):
-        Bn.dlm_token_prob(logits, tok.view(-1), ls, pr)
-        Bn.dlm_refine_update_ranked(tok, msk, am2, cf2, pr2, params, nt, nm, ne)
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-    t_tp = t_up = 0.0
-    for _ in range(reps):
-        ev[0].record(stream)
-        Bn.dlm_token_prob(logits, tok.view(-1), ls, pr)
-        ev[1].record(stream)
-        Bn.dlm_refine_update_ranked(tok, msk, am2, cf2, pr2, params, nt, nm, ne)
-        ev[2].record(stream)
-        torch.cuda.synchronize()
-        t_tp += ev[0].elapsed_time(ev[1])
-        t_up += ev[1].elapsed_time(ev[2])
-    if Bn.device_error(clear=True):
-        raise RuntimeError("device error word set during the ranked-update measurement")
-    return {"token_prob_ms": t_tp / reps, "update_ranked_ms": t_up / reps,
-            "note": "remask ranking by the resulting token's probability (variant reading); not in the step"}
-
-
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -418,12 +388,34 @@ def run_ours(args, rank, world):
     stream = torch.cuda.current_stream(d)
     fused = args.path == "fused"
 
+    ranked = args.rank == "result"
+    if ranked:
+        tprob = torch.empty(w.N, dtype=torch.float32, device=d)
+
+    mask_mode = {"full": 0, "block_causal": 1, "block_local": 2}[args.attn_mask]
+
+    def attention():
+        if mask_mode:
+            Bn.dlm_attn_masked(q, k, v, seqlen, prompt, mask_mode, args.block, out)
+        else:
+            Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+
     def step(ev=None):
         if ev:
             ev[0].record(stream)
-        Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+        attention()
         if ev:
             ev[1].record(stream)
+        if ranked:
+            Bn.dlm_vocab_confidence(logits, am, cf, ls)
+            if ev:
+                ev[2].record(stream)
+            Bn.dlm_token_prob(logits, tok.view(-1), ls, tprob)
+            Bn.dlm_refine_update_ranked(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), tprob.view(w.B, w.L),
+                                        params, nt, nm, ne)
+            if ev:
+                ev[3].record(stream)
+            return
         if fused:
             Bn.dlm_refine_step(logits, tok, msk, params, am.view(w.B, w.L), cf.view(w.B, w.L), ls.view(w.B, w.L),
                                nt, nm, ne, workspace)
@@ -518,12 +510,11 @@ def run_ours(args, rank, world):
 
     # ---- multi-pass refinement: the recorded pass repeated by one graph launch
     # (device-side early stop) against the same passes driven from the host
-    ranked_info = measure_ranked(Bn, w, logits, tok, msk, am, cf, ls, params, stream)
     loop_info = None
     if args.loop_steps > 0:
         loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
 
-    attn_flops = w.attn_flops()
+    attn_flops = w.attn_flops(mask_mode, args.block)
     vocab_bytes = w.vocab_bytes()
     kern = {
         "attn": {"achieved_tflops": attn_flops / (per_kernel["attn"] * 1e-3) / 1e12, "ms": per_kernel["attn"],
@@ -534,6 +525,8 @@ def run_ours(args, rank, world):
     }
     kern["attn"]["frac_of_measured_bf16"] = kern["attn"]["achieved_tflops"] / peaks["bf16_tflops"]
     kern["vocab"]["frac_of_measured_hbm"] = kern["vocab"]["achieved_gbs"] / peaks["hbm_gbs"]
+    if ranked:
+        kern["update"]["kernels"] = "token_prob_kernel + refine_update_kernel (ranking by the resulting token)"
     if fused:   # the vocabulary stream and the update share one launch
         kern["vocab"]["kernel"] = "vocab_step (vocabulary reduction + update)"
         kern["update"] = {"ms": 0.0, "fused_into": "vocab"}
@@ -564,11 +557,12 @@ def run_ours(args, rank, world):
         "refined_tokens_per_sec": steps_per_s * w.refined_tokens(),
         "kernels": kern,
         "roofline": roof,
-        "gpu_launches": (2 if fused else 3) * args.steps,
+        "gpu_launches": (2 if fused else 4 if ranked else 3) * args.steps,
         "path": args.path,
+        "rank": args.rank,
+        "attn_mask": args.attn_mask if not mask_mode else f"{args.attn_mask} (block {args.block})",
         "e2e": e2e,
         "loop": loop_info,
-        "ranked_variant": ranked_info,
     }
     if timer is not None:
         res["cpu_baseline"] = timer.run()
@@ -618,7 +612,15 @@ def main():
     ap.add_argument("--path", default="separate", choices=["fused", "separate"],
                     help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
                          "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")
+    ap.add_argument("--attn-mask", default="full", choices=["full", "block_causal", "block_local"],
+                    help="attention mask of the step (full: the refiner's bidirectional pass)")
+    ap.add_argument("--block", type=int, default=64, help="block size of the block masks")
+    ap.add_argument("--rank", default="conf", choices=["conf", "result"],
+                    help="remask ranking: conf (maximum probability) or result (probability of the token each "
+                         "position ends with: dlm_token_prob + dlm_refine_update_ranked)")
     args = ap.parse_args()
+    if args.rank == "result" and args.path == "fused":
+        ap.error("--rank result runs the separate path")
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     world = int(os.environ.get("WORLD_SIZE", "1"))

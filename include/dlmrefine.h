@@ -119,6 +119,31 @@ typedef struct dlm_refine_params {
 int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v,
                    const dlm_tensor* seq_lens, dlm_tensor* out);
 
+/* Attention masks of dlm_attn_masked. */
+#define DLM_ATTN_FULL 0          /* every valid key (dlm_bidir_attn) */
+#define DLM_ATTN_BLOCK_CAUSAL 1  /* block-autoregressive attention (Sec. 3.3) */
+#define DLM_ATTN_BLOCK_LOCAL 2   /* prompt + own block: local refinement (Sec. 5.3, 6.3) */
+
+/*
+ * dlm_bidir_attn over a subset of keys per query (the block-autoregressive
+ * pattern the refiner replaces, Sec. 3.3, and the local 64-token refinement
+ * of the causal ablation, Sec. 5.3 / 6.3). The response [p_b, n_b) is cut
+ * into blocks of `block` positions starting at p_b; query i >= p_b of block
+ * c = floor((i - p_b) / block) attends to
+ *   DLM_ATTN_BLOCK_CAUSAL  keys j < min(n_b, p_b + (c + 1) * block)
+ *                          (the prompt, earlier blocks and its own block);
+ *   DLM_ATTN_BLOCK_LOCAL   keys j < p_b and keys of block c (j < n_b);
+ * prompt queries i < p_b attend to keys j < p_b. DLM_ATTN_FULL is
+ * dlm_bidir_attn. Rows i >= n_b are 0.
+ *   prompt_lens  [B] I32 (p_b, clamped to [0, n_b]; a clamp sets
+ *                DLM_DEVERR_LENGTH) or NULL (p_b = 0)
+ *   mode         DLM_ATTN_*;  block >= 1 for the block masks
+ *   other arguments as for dlm_bidir_attn (same dtypes, layouts, tolerances).
+ */
+int dlm_attn_masked(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v,
+                    const dlm_tensor* seq_lens, const dlm_tensor* prompt_lens, int32_t mode,
+                    int32_t block, dlm_tensor* out);
+
 /*
  * Step A2 -- per-position reduction over the vocabulary (the confidences the
  * refine threshold of Table 10 and the confident edits of Appendix C.4 act on).

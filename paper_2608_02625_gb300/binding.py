@@ -46,6 +46,7 @@ def _load():
     lib = ctypes.CDLL(library_path)
     P = ctypes.POINTER(DlmTensor)
     lib.dlm_bidir_attn.argtypes = [P, P, P, P, P]
+    lib.dlm_attn_masked.argtypes = [P, P, P, P, P, ctypes.c_int32, ctypes.c_int32, P]
     lib.dlm_vocab_confidence.argtypes = [P, P, P, P]
     lib.dlm_refine_update.argtypes = [P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
     lib.dlm_refine_step.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P,
@@ -55,7 +56,7 @@ def _load():
     lib.dlm_refine_step_static.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P]
     lib.dlm_refine_step_workspace_bytes.argtypes = [ctypes.c_int64]
     lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
-    for f in ("dlm_bidir_attn", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
+    for f in ("dlm_bidir_attn", "dlm_attn_masked", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
               "dlm_refine_step_static", "dlm_token_prob", "dlm_refine_update_ranked", "dlm_set_stream",
               "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
@@ -134,6 +135,19 @@ def dlm_bidir_attn(q, k, v, seq_lens, out):
     _prepare(q, k, v, seq_lens, out)
     dq, dk, dv, ds, do = (describe(t) for t in (q, k, v, seq_lens, out))
     _check(lib.dlm_bidir_attn(_ref(dq), _ref(dk), _ref(dv), _ref(ds), _ref(do)))
+    return out
+
+
+ATTN_FULL, ATTN_BLOCK_CAUSAL, ATTN_BLOCK_LOCAL = 0, 1, 2
+
+
+def dlm_attn_masked(q, k, v, seq_lens, prompt_lens, mode: int, block: int, out):
+    """Attention restricted by a block mask (ATTN_BLOCK_CAUSAL: prompt, earlier
+    blocks and the own block; ATTN_BLOCK_LOCAL: prompt and the own block)."""
+    _prepare(q, k, v, seq_lens, prompt_lens, out)
+    ds = [describe(t) for t in (q, k, v, seq_lens, prompt_lens)]
+    do = describe(out)
+    _check(lib.dlm_attn_masked(*[_ref(d) for d in ds], int(mode), int(block), _ref(do)))
     return out
 
 

@@ -1,6 +1,7 @@
 // Step A1, fp32 path -- non-causal GQA attention on the CUDA cores.
 //
-// Sec. 4.2: every valid position attends to every valid position. fp32
+// Sec. 4.2: every valid position attends to every valid position (the block
+// masks of dlm_attn_masked restrict each query to its key ranges). fp32
 // inputs call for fp32 arithmetic throughout (TF32 tensor cores would not hold
 // a 1e-5 error bound), so this path is a plain online-softmax loop: one warp
 // per query row, lanes split the head dimension, a key's score is a warp
@@ -45,8 +46,19 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) attn_f32_kernel(AttnArgs 
     q[t] = qp[lane + 32 * t] * scale;
     acc[t] = 0.f;
   }
+  int p = 0;
+  if (a.mask_mode != DLM_ATTN_FULL && a.prompt_lens) {
+    p = a.prompt_lens[b];
+    if (p < 0 || p > n) {
+      if (lane == 0) set_device_error(err, DLM_DEVERR_LENGTH);
+      p = p < 0 ? 0 : n;
+    }
+  }
+  const KeyRanges kr = key_ranges(a.mask_mode, a.block, i, n, p);
   float m = -INFINITY, l = 0.f;
-  for (int j = 0; j < n; ++j) {
+  for (int j = 0; j < kr.hi2; ++j) {
+    if (j == kr.hi1 && kr.lo2 > j) j = kr.lo2;   // skip the keys between the two ranges
+    if (j >= kr.hi2) break;
     const float* kj = kb + j * a.sk[1];
     float s = 0.f;
 #pragma unroll

@@ -99,7 +99,9 @@ struct Smem {
 
 struct TcParams {
   int B, L, Hq, Hkv, G, mtiles, units_per_bg, units;
+  int mask_mode, block;
   const int32_t* seq_lens;
+  const int32_t* prompt_lens;
   __nv_bfloat16* out;
   int64_t so0, so1, so2;
   float scale_log2;
@@ -107,11 +109,14 @@ struct TcParams {
 };
 
 struct Unit {
-  int b, g, n, nkv;  // nkv: 64-key sub-tiles
+  int b, g, n, p, nkv;  // nkv: 64-key sub-tiles visited
+  int ka, kgap;         // sub-tile j of the unit is key sub-tile kt(j) = j < ka ? j : j + kgap
   int head[2], row0[2];
   bool active[2], run[2];
+  __device__ __forceinline__ int kt(int j) const { return j < ka ? j : j + kgap; }
 };
 
+template <bool kMasked>
 __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
   Unit U;
   const int bg = unit / p.units_per_bg;
@@ -133,7 +138,41 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
     U.row0[i] = (U.active[i] ? t / p.G : 0) * kTile;
     U.run[i] = U.active[i] && U.row0[i] < n;
   }
-  U.nkv = (U.run[0] || U.run[1]) ? (n + kSub - 1) / kSub : 0;
+  U.p = 0;
+  U.ka = U.nkv = (U.run[0] || U.run[1]) ? (n + kSub - 1) / kSub : 0;
+  U.kgap = 0;
+  if (kMasked && U.nkv > 0) {
+    int pl = p.prompt_lens ? p.prompt_lens[U.b] : 0;
+    if (pl < 0 || pl > n) {
+      if (threadIdx.x == 0) set_device_error(p.err, DLM_DEVERR_LENGTH);
+      pl = pl < 0 ? 0 : n;
+    }
+    U.p = pl;
+    // Key sub-tiles any running row of the unit may use: [0, p) and the span
+    // of the rows' blocks (ranges are monotone in the row).
+    int r_lo = n, r_hi = -1;
+    for (int i = 0; i < 2; ++i) {
+      if (!U.run[i]) continue;
+      r_lo = min(r_lo, U.row0[i]);
+      r_hi = max(r_hi, min(U.row0[i] + kTile, n) - 1);
+    }
+    const KeyRanges lo = key_ranges(p.mask_mode, p.block, r_lo, n, pl);
+    const KeyRanges hi = key_ranges(p.mask_mode, p.block, r_hi, n, pl);
+    if (p.mask_mode == DLM_ATTN_BLOCK_CAUSAL || r_hi < pl) {
+      U.ka = U.nkv = (hi.hi1 + kSub - 1) / kSub;
+    } else {
+      const int a_end = (pl + kSub - 1) / kSub;              // prompt sub-tiles
+      const int c0 = (r_lo < pl ? pl : lo.lo2) / kSub;         // first sub-tile of the lowest block
+      const int c1 = (hi.hi2 + kSub - 1) / kSub;
+      if (c0 <= a_end) {
+        U.ka = U.nkv = max(a_end, c1);
+      } else {
+        U.ka = a_end;
+        U.kgap = c0 - a_end;
+        U.nkv = a_end + (c1 - c0);
+      }
+    }
+  }
   return U;
 }
 
@@ -147,7 +186,9 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, ok);
 }
 
-template <int D>
+// kMasked: the block masks of dlm_attn_masked (a separate instantiation, so
+// that full attention carries none of their per-row bookkeeping).
+template <int D, bool kMasked>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
                    const __grid_constant__ CUtensorMap tv, const __grid_constant__ CUtensorMap to,
@@ -215,13 +256,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto fill = [&](const Unit& U, int j, bool is_v) -> bool {
       const int r = fills % kRing;
       if (fills >= kRing && !warp_wait(&sm.bar_empty[r], ((fills / kRing) - 1) & 1, abort, p.err)) return false;
-      const int valid = U.n - j * kSub;
+      const int key0 = (kMasked ? U.kt(j) : j) * kSub;
+      const int valid = U.n - key0;
       if (!is_v || valid >= kSub) {
         if (lane == 0) {
           mbar_arrive_expect_tx(&sm.bar_full[r], kKvBytes);
           for (int c = 0; c < kBoxes; ++c)
-            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, is_v ? &tv : &tk, &sm.bar_full[r], 64 * c, U.g, j * kSub,
-                        U.b);
+            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, is_v ? &tv : &tk, &sm.bar_full[r], 64 * c, U.g, key0, U.b);
         }
       } else {
         // Last, partial value sub-tile: rows >= n may hold any bit pattern and
@@ -230,7 +271,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
           mbar_arrive_expect_tx(&sm.bar_vtmp, kKvBytes);
           for (int c = 0; c < kBoxes; ++c)
-            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, &tv, &sm.bar_vtmp, 64 * c, U.g, j * kSub, U.b);
+            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, &tv, &sm.bar_vtmp, 64 * c, U.g, key0, U.b);
         }
         ++vtmp;
         if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err)) return false;
@@ -247,7 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       return true;
     };
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
-      const Unit U = decode_unit(p, unit);
+      const Unit U = decode_unit<kMasked>(p, unit);
       if (U.nkv == 0) continue;
       // The unit's first key tiles need only ring slots: start them before
       // the query tiles, which wait for the previous unit's last score MMAs.
@@ -329,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int f = 0;          // ring fills consumed
       bool ok = true;
       for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
-        const Unit U = decode_unit(p, unit);
+        const Unit U = decode_unit<kMasked>(p, unit);
         if (U.nkv == 0) continue;
         const bool run = U.run[i];
         if (run) {
@@ -401,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int units_run = 0;  // bar_o phases consumed
     bool ok = true;
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
-      const Unit U = decode_unit(p, unit);
+      const Unit U = decode_unit<kMasked>(p, unit);
       if (!U.active[i]) continue;
       const int row = U.row0[i] + t;
       if (!U.run[i]) {
@@ -427,6 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_used = -INFINITY;
       float l = 0.f;
       bool pvm_done = false;
+      // This row's keys: [0, hi1) and [lo2, hi2).
+      const KeyRanges kr = kMasked ? key_ranges(p.mask_mode, p.block, row, U.n, U.p) : KeyRanges{U.n, U.n, U.n};
       for (int j = 0; j < U.nkv; ++j) {
         const int b = j & 1;
         const uint32_t s_addr = slot_addr + kSub * b;
@@ -444,11 +487,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         float sv[kSub];
 #pragma unroll
         for (int c = 0; c < kSub; ++c) sv[c] = __uint_as_float(sr[c]);
-        const int valid = U.n - j * kSub;
-        if (valid < kSub) {
+        const int key0 = (kMasked ? U.kt(j) : j) * kSub;
+        if (!(key0 + kSub <= kr.hi1 || (kMasked && key0 >= kr.lo2 && key0 + kSub <= kr.hi2))) {
 #pragma unroll
-          for (int c = 0; c < kSub; ++c)
-            if (c >= valid) sv[c] = -INFINITY;
+          for (int c = 0; c < kSub; ++c) {
+            const int key = key0 + c;
+            if (!(key < kr.hi1 || (kMasked && key >= kr.lo2 && key < kr.hi2))) sv[c] = -INFINITY;
+          }
         }
         float mx0 = sv[0], mx1 = sv[1], mx2 = sv[2], mx3 = sv[3];
 #pragma unroll
@@ -496,7 +541,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Numerators 2^(s * scale - m), two columns at a time; P goes to tensor
         // memory (over the first 32 columns of this S buffer) 16 columns at a time.
         const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
-        const float2 nm2 = make_float2(-m_used, -m_used);
+        // A row whose keys so far were all masked keeps m_used = -inf: its
+        // numerators are exp2(-inf) = 0 (subtracting 0 avoids -inf - -inf).
+        const float m_sub = (kMasked && m_used == -INFINITY) ? 0.f : m_used;
+        const float2 nm2 = make_float2(-m_sub, -m_sub);
         float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
         for (int qq = 0; qq < kSub / 32; ++qq) {
@@ -625,7 +673,7 @@ int make_map(CUtensorMap* map, const void* base, int B, int L, int H, int D, con
   return DLM_OK;
 }
 
-template <int D>
+template <int D, bool kMasked>
 int launch_d(const AttnArgs& a, cudaStream_t stream) {
   CUtensorMap mq, mk, mv, mo;
   int st;
@@ -647,6 +695,9 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   if (units > 0x7FFFFFFFLL) return fail(DLM_ERR_SHAPE, "too many attention work units");
   p.units = static_cast<int>(units);
   p.seq_lens = a.seq_lens;
+  p.prompt_lens = a.prompt_lens;
+  p.mask_mode = a.mask_mode;
+  p.block = a.block > 0 ? a.block : 1;
   p.out = static_cast<__nv_bfloat16*>(a.out);
   p.so0 = a.so[0];
   p.so1 = a.so[1];
@@ -654,14 +705,14 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(D));
   p.err = device_error_word();
   const size_t smem = sizeof(Smem<D>) + 1024;
-  cudaError_t attr_err = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t attr_err = cudaFuncSetAttribute(attn_tc_kernel<D, kMasked>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(smem));
   if (attr_err != cudaSuccess) return fail(DLM_ERR_CUDA, "attn smem attribute: %s", cudaGetErrorString(attr_err));
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = static_cast<int>(units < sms ? units : sms);
-  attn_tc_kernel<D><<<grid, kThreads, smem, stream>>>(mq, mk, mv, mo, p);
+  attn_tc_kernel<D, kMasked><<<grid, kThreads, smem, stream>>>(mq, mk, mv, mo, p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "attn_tc launch: %s", cudaGetErrorString(e));
   return DLM_OK;
@@ -671,7 +722,9 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
 
 int launch_attn_tc_bf16(const AttnArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.L == 0) return DLM_OK;
-  return a.D == 64 ? launch_d<64>(a, stream) : launch_d<128>(a, stream);
+  if (a.mask_mode != DLM_ATTN_FULL)
+    return a.D == 64 ? launch_d<64, true>(a, stream) : launch_d<128, true>(a, stream);
+  return a.D == 64 ? launch_d<64, false>(a, stream) : launch_d<128, false>(a, stream);
 }
 
 }  // namespace dlm

@@ -188,11 +188,17 @@ int dlm_get_device_error(int32_t* bits, int clear) {
   return DLM_OK;
 }
 
-int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v, const dlm_tensor* seq_lens,
-                   dlm_tensor* out) {
+}  // extern "C"
+
+namespace {
+
+int attn_impl(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v, const dlm_tensor* seq_lens,
+              const dlm_tensor* prompt_lens, int32_t mode, int32_t block, dlm_tensor* out) {
   using dlm::fail;
-  t_last_error[0] = '\0';
   int st;
+  if (mode != DLM_ATTN_FULL && mode != DLM_ATTN_BLOCK_CAUSAL && mode != DLM_ATTN_BLOCK_LOCAL)
+    return fail(DLM_ERR_ARG, "unknown attention mask mode %d", mode);
+  if (mode != DLM_ATTN_FULL && block < 1) return fail(DLM_ERR_ARG, "block must be >= 1 for a block mask");
   if ((st = check_tensor(q, "q", kMaskBF16F32, 4, 4))) return st;
   if ((st = check_tensor(k, "k", kMaskBF16F32, 4, 4))) return st;
   if ((st = check_tensor(v, "v", kMaskBF16F32, 4, 4))) return st;
@@ -215,6 +221,11 @@ int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v
     if ((st = check_tensor(seq_lens, "seq_lens", 1 << DLM_I32, 1, 1))) return st;
     if (seq_lens->shape[0] != B) return fail(DLM_ERR_SHAPE, "seq_lens must have B entries");
   }
+  if (prompt_lens) {
+    if ((st = check_tensor(prompt_lens, "prompt_lens", 1 << DLM_I32, 1, 1))) return st;
+    if (prompt_lens->shape[0] != B) return fail(DLM_ERR_SHAPE, "prompt_lens must have B entries");
+    if (overlaps(out, prompt_lens)) return fail(DLM_ERR_ARG, "out overlaps an input");
+  }
   if (overlaps(out, q) || overlaps(out, k) || overlaps(out, v))
     return fail(DLM_ERR_ARG, "out overlaps an input");
   if (B == 0 || L == 0 || Hq == 0) return DLM_OK;
@@ -224,6 +235,9 @@ int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v
   a.v = v->data;
   a.out = out->data;
   a.seq_lens = seq_lens ? static_cast<const int32_t*>(seq_lens->data) : nullptr;
+  a.prompt_lens = prompt_lens && mode != DLM_ATTN_FULL ? static_cast<const int32_t*>(prompt_lens->data) : nullptr;
+  a.mask_mode = mode;
+  a.block = mode != DLM_ATTN_FULL ? block : 1;
   a.B = static_cast<int>(B);
   a.L = static_cast<int>(L);
   a.Hq = static_cast<int>(Hq);
@@ -249,6 +263,22 @@ int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v
   }
   if ((st = require_error_word())) return st;
   return dlm::launch_attn_f32(a, t_stream);
+}
+
+}  // namespace
+
+extern "C" {
+
+int dlm_bidir_attn(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v, const dlm_tensor* seq_lens,
+                   dlm_tensor* out) {
+  t_last_error[0] = '\0';
+  return attn_impl(q, k, v, seq_lens, nullptr, DLM_ATTN_FULL, 1, out);
+}
+
+int dlm_attn_masked(const dlm_tensor* q, const dlm_tensor* k, const dlm_tensor* v, const dlm_tensor* seq_lens,
+                    const dlm_tensor* prompt_lens, int32_t mode, int32_t block, dlm_tensor* out) {
+  t_last_error[0] = '\0';
+  return attn_impl(q, k, v, seq_lens, prompt_lens, mode, block, out);
 }
 
 }  // extern "C"

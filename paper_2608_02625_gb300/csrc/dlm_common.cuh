@@ -64,6 +64,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Wall-clock budget of one bounded wait. Long enough for any legitimate wait
 // inside one launch, short enough that a broken pipeline ends quickly.
+// Keys a query row may attend to under the attention masks of dlmrefine.h:
+// [0, hi1) and [lo2, hi2) (n_b = n, p_b = p clamped to [0, n]).
+struct KeyRanges {
+  int hi1, lo2, hi2;
+};
+
+__host__ __device__ __forceinline__ KeyRanges key_ranges(int mode, int block, int row, int n, int p) {
+  KeyRanges r{n, n, n};
+  if (mode == DLM_ATTN_FULL) return r;
+  if (row < p) {           // prompt queries: the prompt
+    r.hi1 = p;
+    return r;
+  }
+  const int start = p + ((row - p) / block) * block;
+  const int end = start + block < n ? start + block : n;
+  if (mode == DLM_ATTN_BLOCK_CAUSAL) {
+    r.hi1 = end;           // the prompt, earlier blocks and the own block
+  } else {
+    r.hi1 = p;             // the prompt and the own block
+    r.lo2 = start;
+    r.hi2 = end;
+  }
+  return r;
+}
+
 constexpr uint64_t kWaitBudgetNs = 2000000000ull;  // 2 s
 
 // Waits for the phase with parity `parity` of `bar` to complete. Gives up

@@ -25,6 +25,8 @@ struct AttnArgs {
   const void* v;
   void* out;
   const int32_t* seq_lens;  // may be null: n_b = L
+  const int32_t* prompt_lens;  // may be null: p_b = 0 (block masks only)
+  int mask_mode, block;        // DLM_ATTN_* and the block size (block masks)
   int B, L, Hq, Hkv, D;
   // strides in elements, (b, l, h) order; the innermost stride is 1
   int64_t sq[3], sk[3], sv[3], so[3];

@@ -16,6 +16,19 @@ import numpy as np
 from . import synth
 
 
+def attended_pairs(n: int, p: int, mask_mode: int, block: int) -> int:
+    """(query, key) pairs a sequence of n positions (prompt p) attends to under
+    an attention mask: 0 full, 1 block-causal, 2 block-local (dlmrefine.h)."""
+    if mask_mode == 0:
+        return n * n
+    p = min(max(p, 0), n)
+    i = np.arange(p, n)
+    start = p + ((i - p) // block) * block
+    end = np.minimum(n, start + block)
+    own = end if mask_mode == 1 else p + (end - start)
+    return int(p * p + own.sum())
+
+
 @dataclasses.dataclass(frozen=True)
 class Workload:
     name: str
@@ -78,10 +91,12 @@ class Workload:
         tok = np.where(m == 1, self.mask_id, tok).astype(np.int32)
         return tok, m
 
-    def attn_flops(self) -> float:
-        """Algorithmic FLOPs of one attention call: sum_b 4 * Hq * n_b^2 * D."""
-        n = self.seq_lens().astype(np.float64)
-        return float(np.sum(4.0 * self.Hq * n * n * self.D))
+    def attn_flops(self, mask_mode: int = 0, block: int = 64) -> float:
+        """Algorithmic FLOPs of one attention call: 4 * Hq * D per attended
+        (query, key) pair; sum_b 4 * Hq * n_b^2 * D without a mask."""
+        pairs = sum(attended_pairs(int(n), int(p), mask_mode, block)
+                    for n, p in zip(self.seq_lens(), self.prompt_lens()))
+        return float(4.0 * self.Hq * self.D * pairs)
 
     def logit_bytes(self) -> int:
         esz = 2 if self.dtype == "bf16" else 4

@@ -301,3 +301,14 @@ def test_update_ranked_rejects(case, status):
     r = lambda x: ctypes.byref(x) if x is not None else None
     assert lib.dlm_refine_update_ranked(r(d["tok"]), r(d["msk"]), r(d["am"]), r(d["cf"]), r(d["tp"]), r(P()),
                                         r(d["nt"]), r(d["nm"]), r(d["ne"])) == status
+
+
+def test_masked_attention_rejects():
+    from paper_2608_02625_gb300.binding import lib
+    q, k, v, sl, o = good_attn()
+    pl = T(I32, [2], 6 * MB)
+    r = ctypes.byref
+    assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(pl), 3, 64, r(o)) == -6         # unknown mode
+    assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(pl), 1, 0, r(o)) == -6          # block < 1
+    assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(T(I32, [3], 6 * MB)), 1, 64, r(o)) == -3
+    assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(T(F32, [2], 6 * MB)), 2, 64, r(o)) == -2
