@@ -22,6 +22,10 @@ which any response position may be revised. One pass on the hot path is
   optionally ranked by the probability of each position's resulting token,
   with ``vocab.token_prob`` giving the probability of a kept token.
 
+``lmhead.lm_head_confidence`` is the vocabulary projection (hidden states times
+the output weights) followed by ``vocab.vocab_confidence``, the operation of
+the fused projection + reduction kernel.
+
 Floating point is fp64 unless a comparison is defined in fp32 (edit threshold,
 remask order), where the fp32 values are compared exactly.
 
@@ -32,3 +36,4 @@ forms, invariants and hand-worked update examples (tests/golden/).
 from .attention import bidir_attn  # noqa: F401
 from .vocab import token_prob, vocab_confidence  # noqa: F401
 from .update import refine_update, remask_count  # noqa: F401
+from .lmhead import lm_head_confidence, lm_head_logits  # noqa: F401

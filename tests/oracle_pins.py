@@ -332,8 +332,54 @@ def pin_token_prob_torch():
     assert abs(tot - 1.0) <= 1e-5
 
 
+def pin_lmhead_brute_force():
+    """Tiny case with explicit dot products and a max / sum written out."""
+    rng = np.random.default_rng(25)
+    h = rng.standard_normal((3, 5))
+    w = rng.standard_normal((7, 5))
+    am, conf, lse = oracle.lm_head_confidence(h, w)
+    for r in range(3):
+        x = [sum(h[r, k] * w[v, k] for k in range(5)) for v in range(7)]
+        mx = max(x)
+        S = sum(math.exp(t - mx) for t in x)
+        assert am[r] == x.index(mx)
+        assert abs(float(lse[r]) - (mx + math.log(S))) <= 1e-6 * max(1.0, abs(mx))
+        assert abs(float(conf[r]) - 1.0 / S) <= 1e-6 / S
+
+
+def pin_lmhead_torch():
+    """torch fp64 matmul + logsumexp / softmax / argmax, with the vocabulary
+    spread over several projection blocks."""
+    rng = np.random.default_rng(26)
+    h = rng.standard_normal((9, 64))
+    w = rng.standard_normal((3000, 64)) / 8.0
+    logits = oracle.lm_head_logits(h, w, block=1000)
+    t = torch.from_numpy(h) @ torch.from_numpy(w).T
+    assert np.abs(logits - t.numpy()).max() <= 1e-12
+    am, conf, lse = oracle.lm_head_confidence(h, w)
+    assert np.array_equal(am, torch.argmax(t, dim=1).numpy())
+    assert np.all(np.abs(lse - torch.logsumexp(t, 1).numpy()) <= 1e-6 * np.abs(lse))
+    c = torch.softmax(t, 1).max(1).values.numpy()
+    assert np.all(np.abs(conf - c) <= 1e-6 * c)
+
+
+def pin_lmhead_one_hot_weights():
+    """Weight rows that pick single hidden coordinates: the logits are those
+    coordinates, so the reduction of the projection is the reduction of the
+    selected columns."""
+    rng = np.random.default_rng(27)
+    h = rng.standard_normal((4, 6))
+    sel = np.array([5, 0, 3, 3, 1])
+    w = np.eye(6)[sel]
+    got = oracle.lm_head_confidence(h, w)
+    ref = oracle.vocab_confidence(h[:, sel])
+    for a, b in zip(got, ref):
+        assert np.array_equal(a, b)
+
+
 VOCAB_PINS = [pin_vocab_uniform_row, pin_vocab_single_finite, pin_vocab_two_valued_closed_form,
-              pin_vocab_ties_lowest_index, pin_vocab_torch, pin_token_prob_closed_forms, pin_token_prob_torch]
+              pin_vocab_ties_lowest_index, pin_vocab_torch, pin_token_prob_closed_forms, pin_token_prob_torch,
+              pin_lmhead_brute_force, pin_lmhead_torch, pin_lmhead_one_hot_weights]
 
 
 # ---------------------------------------------------------------- update

@@ -6,7 +6,7 @@ last instead of the first maximum, a strict threshold, ties broken towards the
 higher index, a rounded-up remask count, a block-causal mask that drops the
 query's own block, a block-local mask without the prompt, a resulting-token ranking that
 ignores which positions end with their argmax, a sign slip in a token's
-probability. If a pin suite let one through, the
+probability, a projection that pairs the wrong feature indices. If a pin suite let one through, the
 oracle could carry that slip undetected."""
 import math
 
@@ -16,6 +16,7 @@ import pytest
 import oracle_pins as P
 from oracle import attention as oatt
 from oracle import update as oupd
+from oracle import lmhead as olmh
 from oracle import vocab as ovoc
 
 MUTATIONS = {
@@ -40,6 +41,7 @@ MUTATIONS = {
                         lambda cv, pos: sorted(pos, key=lambda i: (cv[i], -i)), P.UPDATE_PINS),
     "result_rank_ignores_argmax": (oupd, "resulting_token_prob", lambda nt, pred, c, tp: tp, P.UPDATE_PINS),
     "token_prob_sign": (ovoc, "softmax_prob", lambda x, lse: float(np.exp(lse - x)), P.VOCAB_PINS),
+    "projection_reversed_features": (olmh, "project", lambda h, w: h @ w[:, ::-1].T, P.VOCAB_PINS),
     "ceil_remask_count": (oupd, "remask_count",
                           lambda k, f, r: max(0, min(k if k >= 0 else
                                                      math.ceil(float(np.float32(f)) * r), r)),
