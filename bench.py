@@ -348,6 +348,62 @@ def measure_loop(args, w, Bn, q, k, v, out, logits, tok0, msk0, params, seqlen, 
                     "graph: CUDA events around one launch; host-driven: wall clock, one n_edits read-back per pass"}
 
 
+def measure_lmhead(args, w, Bn, peaks, reps=10):
+    """The vocabulary projection fused with the reduction (dlm_lmhead_confidence)
+    on the workload's N rows and V tokens at width d = --lmhead-d, against the
+    unfused pair: a cuBLAS bf16 GEMM writing the bf16 logits (torch.matmul)
+    followed by dlm_vocab_confidence. Inputs: seeded normals on the device."""
+    import torch
+    from paper_2608_02625_gb300 import synth, synth_gpu
+    d = torch.device("cuda", torch.cuda.current_device())
+    dm = args.lmhead_d
+    hidden = torch.empty((w.N, dm), dtype=torch.bfloat16, device=d)
+    weight = torch.empty((w.V, dm), dtype=torch.bfloat16, device=d)
+    synth_gpu.fill_normal_(hidden, synth.stream_key(w.seed + 101, synth.S_Q), 1.0)
+    synth_gpu.fill_normal_(weight, synth.stream_key(w.seed + 101, synth.S_K), 1.0 / dm ** 0.5)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    ws = torch.empty(Bn.dlm_lmhead_workspace_bytes(w.N), dtype=torch.uint8, device=d)
+    stream = torch.cuda.current_stream(d)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    t_fused = timed(lambda: Bn.dlm_lmhead_confidence(hidden, weight, am, cf, ls, ws))
+    am_f = am.clone()
+    logits = torch.empty((w.N, w.V), dtype=torch.bfloat16, device=d)
+
+    def unfused():
+        torch.matmul(hidden, weight.t(), out=logits)
+        Bn.dlm_vocab_confidence(logits, am, cf, ls)
+
+    t_unfused = timed(unfused)
+    t_gemm = timed(lambda: torch.matmul(hidden, weight.t(), out=logits))
+    agree = float((am == am_f).float().mean().item())
+    del logits
+    torch.cuda.empty_cache()
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the projection measurement")
+    flops = 2.0 * w.N * w.V * dm
+    return {"rows": w.N, "vocab": w.V, "d": dm, "flops": flops, "ms_fused": t_fused,
+            "tflops_fused": flops / (t_fused * 1e-3) / 1e12,
+            "frac_of_measured_bf16": flops / (t_fused * 1e-3) / 1e12 / peaks["bf16_tflops"],
+            "ms_unfused_gemm_plus_vocab": t_unfused, "ms_cublas_gemm_alone": t_gemm,
+            "argmax_agreement_fused_vs_unfused": agree,
+            "note": "unfused = torch.matmul (cuBLAS, bf16 logits written) + dlm_vocab_confidence; "
+                    "the fused kernel keeps fp32 logits, so argmax agreement below 1 is near-ties and bf16 rounding"}
+
+
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -510,6 +566,7 @@ def run_ours(args, rank, world):
 
     # ---- multi-pass refinement: the recorded pass repeated by one graph launch
     # (device-side early stop) against the same passes driven from the host
+    lmhead_info = measure_lmhead(args, w, Bn, peaks) if args.lmhead_d > 0 else None
     loop_info = None
     if args.loop_steps > 0:
         loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
@@ -563,6 +620,7 @@ def run_ours(args, rank, world):
         "attn_mask": args.attn_mask if not mask_mode else f"{args.attn_mask} (block {args.block})",
         "e2e": e2e,
         "loop": loop_info,
+        "lmhead": lmhead_info,
     }
     if timer is not None:
         res["cpu_baseline"] = timer.run()
@@ -612,6 +670,8 @@ def main():
     ap.add_argument("--path", default="separate", choices=["fused", "separate"],
                     help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
                          "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")
+    ap.add_argument("--lmhead-d", type=int, default=2048,
+                    help="also time the vocabulary projection fused with the reduction at this width (0: skip)")
     ap.add_argument("--attn-mask", default="full", choices=["full", "block_causal", "block_local"],
                     help="attention mask of the step (full: the refiner's bidirectional pass)")
     ap.add_argument("--block", type=int, default=64, help="block size of the block masks")

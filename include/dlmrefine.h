@@ -89,6 +89,10 @@ typedef struct dlm_tensor {
  *   prompt_lens     device int32[B]: p_b, clamped into [0, n_b].
  *   seq_lens        device int32[B]: n_b, clamped into [0, L].
  * The response of sequence b is [p_b, n_b) and r_b = n_b - p_b.
+ * The update only touches [p_b, n_b): to refine one window of a response
+ * (the local 64-token refinement of Sec. 6.3 and the granular span schedules
+ * of Appendix D.4), pass the window's bounds here (the attention keeps the
+ * sequence's own lengths); positions outside the window are copied unchanged.
  */
 typedef struct dlm_refine_params {
   float edit_threshold;
@@ -187,6 +191,30 @@ int dlm_vocab_confidence(const dlm_tensor* logits, dlm_tensor* argmax, dlm_tenso
 int dlm_refine_update(const dlm_tensor* tokens, const dlm_tensor* mask, const dlm_tensor* argmax,
                       const dlm_tensor* conf, const dlm_refine_params* params,
                       dlm_tensor* new_tokens, dlm_tensor* new_mask, dlm_tensor* n_edits);
+
+/*
+ * The vocabulary projection fused with step A2: for each row r of hidden,
+ * the per-position reduction of dlm_vocab_confidence applied to
+ *   logits[r, v] = sum_k hidden[r, k] * weight[v, k]      (v < V),
+ * the refiner's output projection of its final hidden states (Sec. 4.2: every
+ * revisable position's distribution over the vocabulary), without writing
+ * the N x V logits to memory. tcgen05 MMAs (bf16 x bf16, fp32 accumulation);
+ * the reduction reads the fp32 accumulators (no bf16 rounding of logits).
+ *   hidden     [N, d] or [B, L, d] BF16, weight [V, d] BF16; d a multiple of
+ *              64; base pointers and row strides multiples of 16 bytes
+ *   argmax, conf, lse   N entries each (I32, F32, F32), contiguous
+ *   workspace  >= dlm_lmhead_workspace_bytes(N) bytes of device memory,
+ *              16-byte aligned, owned by the caller (no initial contents
+ *              needed); calls sharing it must not overlap on the GPU.
+ * Accuracy: the logits carry fp32 accumulation error (a few 1e-5 relative to
+ * sum_k |hidden[r,k] weight[v,k]|); an argmax can differ from exact
+ * arithmetic only where two logits are that close. The width d is a
+ * parameter: the paper does not give the refiner's dimensions.
+ */
+int dlm_lmhead_confidence(const dlm_tensor* hidden, const dlm_tensor* weight, dlm_tensor* argmax,
+                          dlm_tensor* conf, dlm_tensor* lse, void* workspace, size_t workspace_bytes);
+/* Bytes of workspace dlm_lmhead_confidence needs for `rows` rows. */
+size_t dlm_lmhead_workspace_bytes(int64_t rows);
 
 /*
  * Probability of a given token of each row under the row's softmax:

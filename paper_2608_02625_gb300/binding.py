@@ -52,12 +52,16 @@ def _load():
     lib.dlm_refine_step.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P,
                                     ctypes.c_void_p, ctypes.c_size_t]
     lib.dlm_token_prob.argtypes = [P, P, P, P]
+    lib.dlm_lmhead_confidence.argtypes = [P, P, P, P, P, ctypes.c_void_p, ctypes.c_size_t]
+    lib.dlm_lmhead_workspace_bytes.argtypes = [ctypes.c_int64]
+    lib.dlm_lmhead_workspace_bytes.restype = ctypes.c_size_t
     lib.dlm_refine_update_ranked.argtypes = [P, P, P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P]
     lib.dlm_refine_step_static.argtypes = [P, P, P, ctypes.POINTER(DlmRefineParams), P, P, P, P, P, P]
     lib.dlm_refine_step_workspace_bytes.argtypes = [ctypes.c_int64]
     lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
     for f in ("dlm_bidir_attn", "dlm_attn_masked", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
-              "dlm_refine_step_static", "dlm_token_prob", "dlm_refine_update_ranked", "dlm_set_stream",
+              "dlm_refine_step_static", "dlm_token_prob", "dlm_refine_update_ranked", "dlm_lmhead_confidence",
+              "dlm_set_stream",
               "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
     lib.dlm_loop_begin.argtypes = [ctypes.c_void_p]
@@ -184,6 +188,22 @@ def dlm_refine_update(tokens, mask, argmax, conf, params: RefineParams, new_toke
     cp = params.to_c()
     _check(lib.dlm_refine_update(*[_ref(d) for d in ds], ctypes.byref(cp), *[_ref(d) for d in outs]))
     return new_tokens, new_mask, n_edits
+
+
+def dlm_lmhead_workspace_bytes(rows: int) -> int:
+    return lib.dlm_lmhead_workspace_bytes(int(rows))
+
+
+def dlm_lmhead_confidence(hidden, weight, argmax, conf, lse, workspace):
+    """argmax / conf / lse of hidden @ weight^T per row, without materialising the logits."""
+    _prepare(hidden, weight, argmax, conf, lse, workspace)
+    if not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
+    ds = [describe(t) for t in (hidden, weight, argmax, conf, lse)]
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(lib.dlm_lmhead_confidence(*[_ref(d) for d in ds], ctypes.c_void_p(workspace.data_ptr() if nbytes else None),
+                                     ctypes.c_size_t(nbytes)))
+    return argmax, conf, lse
 
 
 def dlm_token_prob(logits, tokens, lse, prob):

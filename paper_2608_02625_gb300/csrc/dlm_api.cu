@@ -494,6 +494,73 @@ int dlm_refine_update_ranked(const dlm_tensor* tokens, const dlm_tensor* mask, c
   return dlm::launch_refine_update(a, t_stream);
 }
 
+size_t dlm_lmhead_workspace_bytes(int64_t rows) { return rows > 0 ? dlm::lmhead_workspace_bytes(rows) : 0; }
+
+int dlm_lmhead_confidence(const dlm_tensor* hidden, const dlm_tensor* weight, dlm_tensor* argmax, dlm_tensor* conf,
+                          dlm_tensor* lse, void* workspace, size_t workspace_bytes) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  int st;
+  if ((st = check_tensor(hidden, "hidden", 1 << DLM_BF16, 2, 3))) return st;
+  if ((st = check_tensor(weight, "weight", 1 << DLM_BF16, 2, 2))) return st;
+  if ((st = check_tensor(argmax, "argmax", 1 << DLM_I32, 1, 3))) return st;
+  if ((st = check_tensor(conf, "conf", 1 << DLM_F32, 1, 3))) return st;
+  if ((st = check_tensor(lse, "lse", 1 << DLM_F32, 1, 3))) return st;
+  const int nd = hidden->ndim;
+  const int64_t d = hidden->shape[nd - 1];
+  int64_t N = 1;
+  for (int i = 0; i < nd - 1; ++i) N *= hidden->shape[i];
+  const int64_t V = weight->shape[0];
+  const int64_t s_hidden = hidden->stride[nd - 2];
+  if (nd == 3 && hidden->shape[0] > 1 && hidden->shape[1] > 1 && hidden->stride[0] != hidden->shape[1] * s_hidden)
+    return fail(DLM_ERR_STRIDE, "3-D hidden must be [B, L, d] with evenly strided rows");
+  if (weight->shape[1] != d) return fail(DLM_ERR_SHAPE, "weight must be [V, d] with the d of hidden");
+  if (d < 64 || d % 64 != 0) return fail(DLM_ERR_SHAPE, "d must be a positive multiple of 64 (got %lld)", (long long)d);
+  if (V < 1 && N > 0) return fail(DLM_ERR_SHAPE, "V must be >= 1");
+  if (N > 0x7FFFFFFFLL || V > 0x7FFFFFFFLL) return fail(DLM_ERR_SHAPE, "N and V must be < 2^31");
+  const dlm_tensor* mats[2] = {hidden, weight};
+  for (const dlm_tensor* t : mats) {
+    if (numel(t) == 0) continue;
+    if (reinterpret_cast<uintptr_t>(t->data) % 16 != 0) return fail(DLM_ERR_ALIGN, "hidden / weight not 16-byte aligned");
+    for (int i = 0; i < t->ndim - 1; ++i)
+      if ((t->stride[i] * 2) % 16 != 0) return fail(DLM_ERR_ALIGN, "hidden / weight strides must be multiples of 16 bytes");
+  }
+  const dlm_tensor* outs[3] = {argmax, conf, lse};
+  for (const dlm_tensor* t : outs) {
+    if (numel(t) != N) return fail(DLM_ERR_SHAPE, "argmax, conf and lse must have one entry per row of hidden");
+    if (!is_dense(t)) return fail(DLM_ERR_STRIDE, "argmax, conf and lse must be contiguous");
+    if (overlaps(t, hidden) || overlaps(t, weight)) return fail(DLM_ERR_ARG, "an output overlaps an input");
+  }
+  if (overlaps(argmax, conf) || overlaps(argmax, lse) || overlaps(conf, lse))
+    return fail(DLM_ERR_ARG, "outputs overlap each other");
+  if (N == 0) return DLM_OK;
+  if (!workspace) return fail(DLM_ERR_NULL, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0) return fail(DLM_ERR_ALIGN, "workspace not 16-byte aligned");
+  const size_t need = dlm::lmhead_workspace_bytes(N);
+  if (workspace_bytes < need) return fail(DLM_ERR_ARG, "workspace too small: %zu bytes, %zu needed", workspace_bytes, need);
+  const uintptr_t wlo = reinterpret_cast<uintptr_t>(workspace), whi = wlo + need;
+  const dlm_tensor* all[5] = {hidden, weight, argmax, conf, lse};
+  for (const dlm_tensor* t : all) {
+    uintptr_t lo, hi;
+    byte_span(t, &lo, &hi);
+    if (numel(t) > 0 && lo < whi && wlo < hi) return fail(DLM_ERR_ARG, "workspace overlaps a tensor");
+  }
+  if ((st = require_error_word())) return st;
+  dlm::LmArgs a;
+  a.hidden = hidden->data;
+  a.weight = weight->data;
+  a.N = N;
+  a.V = V;
+  a.d = d;
+  a.s_hidden = N > 1 ? s_hidden : d;
+  a.s_weight = V > 1 ? weight->stride[0] : d;
+  a.argmax = static_cast<int32_t*>(argmax->data);
+  a.conf = static_cast<float*>(conf->data);
+  a.lse = static_cast<float*>(lse->data);
+  a.workspace = workspace;
+  return dlm::launch_lmhead(a, t_stream);
+}
+
 size_t dlm_refine_step_workspace_bytes(int64_t batch) {
   return batch > 0 ? static_cast<size_t>(batch) * sizeof(int32_t) : 0;
 }

@@ -78,4 +78,21 @@ int launch_token_prob(const VocabArgs& a, const int32_t* tokens, const float* ls
 // u.argmax / u.conf alias a.argmax / a.conf). counters: int32[B], zero on entry.
 int launch_vocab_step(const VocabArgs& a, const UpdateArgs& u, int* counters, cudaStream_t stream);
 
+// Vocabulary projection fused with the reduction: per row r of hidden [N, d]
+// the argmax / conf / lse of hidden[r] . weight[v] over v < V.
+struct LmArgs {
+  const void* hidden;   // bf16 [N, d], row stride s_hidden elements
+  const void* weight;   // bf16 [V, d], row stride s_weight elements
+  int64_t N, V, d, s_hidden, s_weight;
+  int32_t* argmax;
+  float* conf;
+  float* lse;
+  void* workspace;      // lmhead_workspace_bytes(N)
+};
+
+constexpr int kLmMaxSplits = 64;
+inline size_t lmhead_workspace_bytes(int64_t N) { return static_cast<size_t>(N) * kLmMaxSplits * 12; }
+int lmhead_splits(int64_t N, int64_t V, int sms);
+int launch_lmhead(const LmArgs& a, cudaStream_t stream);
+
 }  // namespace dlm

@@ -104,3 +104,25 @@ def test_length_clamp_sets_error_word():
     assert_same(gpu, ref, "clamped")
     assert Bn.device_error(clear=True) & 0x1
     assert Bn.device_error(clear=True) == 0
+
+
+@pytest.mark.parametrize("lo,hi", [(0, 64), (64, 128), (300, 512), (100, 101)])
+def test_editable_window(lo, hi):
+    """Refining one window [p_b + lo, p_b + hi) of each response: the window's
+    bounds go in prompt_lens / seq_lens. Inside it the rules apply as to a
+    response (against the oracle with the same bounds); everything outside,
+    masked positions included, is unchanged."""
+    rng = np.random.default_rng(lo * 7 + hi)
+    B, L, V = 4, 640, 1000
+    case = P.random_update_case(rng, B=B, L=L, V=V)
+    p = np.array([256, 128, 0, 600]); n = np.array([640, 500, 640, 640])
+    wlo = np.minimum(n, p + lo); whi = np.minimum(n, p + hi)
+    ref = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"], edit_threshold=0.5,
+                               remask_k=3, remask_frac=0.0, mask_id=V, prompt_lens=wlo, seq_lens=whi)
+    gpu = run_gpu(case["tokens"], case["mask"], case["argmax"], case["conf"], tau=0.5, k=3, frac=0.0, mask_id=V,
+                  prompt=wlo, seqlen=whi)
+    assert_same(gpu, ref, f"window [{lo}, {hi})")
+    for b in range(B):
+        out = np.r_[0:wlo[b], whi[b]:L]
+        assert np.array_equal(gpu[0][b, out], case["tokens"][b, out])
+        assert np.array_equal(gpu[1][b, out], case["mask"][b, out])
