@@ -404,6 +404,138 @@ def measure_lmhead(args, w, Bn, peaks, reps=10):
                     "the fused kernel keeps fp32 logits, so argmax agreement below 1 is near-ties and bf16 rounding"}
 
 
+def build_step(Bn, w, bufs, args, stream, mask_mode):
+    """One refine step on the device buffers in `bufs` (q, k, v, logits, tok,
+    msk, prompt, seqlen); adds its outputs and scratch to `bufs`. step(ev)
+    records ev[0..3] around attention, the vocabulary reduction and the update."""
+    import torch
+    d = bufs["q"].device
+    q, k, v, logits, tok, msk = (bufs[n] for n in ("q", "k", "v", "logits", "tok", "msk"))
+    prompt, seqlen = bufs["prompt"], bufs["seqlen"]
+    out = torch.empty_like(q)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
+    workspace = torch.zeros(Bn.dlm_refine_step_workspace_bytes(w.B) // 4, dtype=torch.int32, device=d)
+    tprob = torch.empty(w.N, dtype=torch.float32, device=d) if args.rank == "result" else None
+    bufs.update(out=out, am=am, cf=cf, ls=ls, nt=nt, nm=nm, ne=ne, params=params)
+
+    def rec(ev, i):
+        if ev:
+            ev[i].record(stream)
+
+    def step(ev=None):
+        rec(ev, 0)
+        if mask_mode:
+            Bn.dlm_attn_masked(q, k, v, seqlen, prompt, mask_mode, args.block, out)
+        else:
+            Bn.dlm_bidir_attn(q, k, v, seqlen, out)
+        rec(ev, 1)
+        if args.path == "fused":
+            Bn.dlm_refine_step(logits, tok, msk, params, am.view(w.B, w.L), cf.view(w.B, w.L), ls.view(w.B, w.L),
+                               nt, nm, ne, workspace)
+            rec(ev, 2)
+            rec(ev, 3)
+            return
+        Bn.dlm_vocab_confidence(logits, am, cf, ls)
+        rec(ev, 2)
+        if tprob is not None:
+            Bn.dlm_token_prob(logits, tok.view(-1), ls, tprob)
+            Bn.dlm_refine_update_ranked(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), tprob.view(w.B, w.L),
+                                        params, nt, nm, ne)
+        else:
+            Bn.dlm_refine_update(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), params, nt, nm, ne)
+        rec(ev, 3)
+
+    return step
+
+
+def measure_e2e(args, Bn, w, bufs, stream, mask_mode, world, d, copy_streams=4):
+    """The same step end to end with HOST inputs: every step copies its inputs
+    from pinned host memory and reads its outputs back, inside the timed
+    region. Two device input sets alternate, so the copies of step s + 1
+    (split over several copy streams, one DMA engine each) overlap the compute
+    of step s; the compute of a step waits for its own copies."""
+    import torch
+    names = ("q", "k", "v", "logits", "tok", "msk", "prompt", "seqlen")
+    host = {}
+    for n in names:
+        t = torch.empty(bufs[n].shape, dtype=bufs[n].dtype, pin_memory=True)
+        t.copy_(bufs[n])
+        host[n] = t
+    sets = [bufs, {n: torch.empty_like(bufs[n]) for n in names}]
+    steps = [None, None]
+    steps[0] = build_step(Bn, w, sets[0], args, stream, mask_mode)   # new outputs for the e2e leg
+    steps[1] = build_step(Bn, w, sets[1], args, stream, mask_mode)
+    outs = ("nt", "nm", "ne")
+    h_out = [{n: torch.empty(sets[i][n].shape, dtype=sets[i][n].dtype, pin_memory=True) for n in outs}
+             for i in range(2)]
+    h2d = sum(host[n].numel() * host[n].element_size() for n in names)
+    d2h = sum(h_out[0][n].numel() * h_out[0][n].element_size() for n in outs)
+    cstreams = [torch.cuda.Stream(d) for _ in range(copy_streams)]
+    free = [torch.cuda.Event(), torch.cuda.Event()]
+    free_recorded = [False, False]
+
+    def copy_in(i):
+        """Issue the host -> device copies of set i; returns the events the compute must wait for."""
+        evs = []
+        for c, cs in enumerate(cstreams):
+            if free_recorded[i]:
+                cs.wait_event(free[i])   # the set's previous step has consumed it
+            with torch.cuda.stream(cs):
+                for n in names:
+                    src, dst = host[n], sets[i][n]
+                    rows = src.shape[0]
+                    if src.numel() * src.element_size() < (64 << 20):
+                        if c == 0:
+                            dst.copy_(src, non_blocking=True)
+                        continue
+                    lo, hi = rows * c // len(cstreams), rows * (c + 1) // len(cstreams)
+                    dst[lo:hi].copy_(src[lo:hi], non_blocking=True)
+            e = torch.cuda.Event()
+            e.record(cs)
+            evs.append(e)
+        return evs
+
+    def run(nsteps):
+        pending = copy_in(0)
+        for s in range(nsteps):
+            i = s & 1
+            for e in pending:
+                stream.wait_event(e)
+            if s + 1 < nsteps:
+                nxt = copy_in(1 - i)          # overlaps this step's compute
+            steps[i]()
+            free[i].record(stream)
+            free_recorded[i] = True
+            for n in outs:
+                h_out[i][n].copy_(sets[i][n], non_blocking=True)
+            if s + 1 < nsteps:
+                pending = nxt
+
+    run(2)
+    torch.cuda.synchronize()
+    k_e2e = max(4, min(args.steps, 20))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    run(k_e2e)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    te = max_over_ranks(e0.elapsed_time(e1) / k_e2e, world, d)
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the end-to-end measurement")
+    return {"value": job_steps_per_s(te, world), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": te, "steps": k_e2e,
+            "copies": f"{copy_streams} copy streams, two device input sets (copies of step s+1 overlap step s)"}
+
+
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -433,58 +565,13 @@ def run_ours(args, rank, world):
     logits = synth_gpu.logits(w, 0, d, tok.view(-1), msk.view(-1))
     prompt = torch.from_numpy(w.prompt_lens()).to(d)
     seqlen = torch.from_numpy(w.seq_lens()).to(d)
-    out = torch.empty_like(q)
-    am = torch.empty(w.N, dtype=torch.int32, device=d)
-    cf = torch.empty(w.N, dtype=torch.float32, device=d)
-    ls = torch.empty(w.N, dtype=torch.float32, device=d)
-    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
-    ne = torch.empty(w.B, dtype=torch.int32, device=d)
-    params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
-    workspace = torch.zeros(Bn.dlm_refine_step_workspace_bytes(w.B) // 4, dtype=torch.int32, device=d)
     stream = torch.cuda.current_stream(d)
     fused = args.path == "fused"
-
     ranked = args.rank == "result"
-    if ranked:
-        tprob = torch.empty(w.N, dtype=torch.float32, device=d)
-
     mask_mode = {"full": 0, "block_causal": 1, "block_local": 2}[args.attn_mask]
-
-    def attention():
-        if mask_mode:
-            Bn.dlm_attn_masked(q, k, v, seqlen, prompt, mask_mode, args.block, out)
-        else:
-            Bn.dlm_bidir_attn(q, k, v, seqlen, out)
-
-    def step(ev=None):
-        if ev:
-            ev[0].record(stream)
-        attention()
-        if ev:
-            ev[1].record(stream)
-        if ranked:
-            Bn.dlm_vocab_confidence(logits, am, cf, ls)
-            if ev:
-                ev[2].record(stream)
-            Bn.dlm_token_prob(logits, tok.view(-1), ls, tprob)
-            Bn.dlm_refine_update_ranked(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), tprob.view(w.B, w.L),
-                                        params, nt, nm, ne)
-            if ev:
-                ev[3].record(stream)
-            return
-        if fused:
-            Bn.dlm_refine_step(logits, tok, msk, params, am.view(w.B, w.L), cf.view(w.B, w.L), ls.view(w.B, w.L),
-                               nt, nm, ne, workspace)
-            if ev:
-                ev[2].record(stream)
-                ev[3].record(stream)
-            return
-        Bn.dlm_vocab_confidence(logits, am, cf, ls)
-        if ev:
-            ev[2].record(stream)
-        Bn.dlm_refine_update(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), params, nt, nm, ne)
-        if ev:
-            ev[3].record(stream)
+    bufs = dict(q=q, k=k, v=v, logits=logits, tok=tok, msk=msk, prompt=prompt, seqlen=seqlen)
+    step = build_step(Bn, w, bufs, args, stream, mask_mode)
+    out, params = bufs["out"], bufs["params"]
 
     clk = ClockSampler(d.index if d.index is not None else 0).__enter__()
     for _ in range(args.warmup):
@@ -521,45 +608,8 @@ def run_ours(args, rank, world):
     ms_per_step = total_ms / args.steps
 
     # ---- end to end through the public API with host buffers
-    e2e = None
-    if not args.no_e2e:
-        h_q, h_k, h_v = q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory()
-        h_logits = torch.empty(logits.shape, dtype=logits.dtype, pin_memory=True)
-        h_logits.copy_(logits)
-        h_tok, h_msk = tok.cpu().pin_memory(), msk.cpu().pin_memory()
-        h_p, h_n = prompt.cpu().pin_memory(), seqlen.cpu().pin_memory()
-        o_tok = torch.empty(tok.shape, dtype=tok.dtype, pin_memory=True)
-        o_msk = torch.empty(msk.shape, dtype=msk.dtype, pin_memory=True)
-        o_ne = torch.empty(ne.shape, dtype=ne.dtype, pin_memory=True)
-        ins = [(h_q, q), (h_k, k), (h_v, v), (h_logits, logits), (h_tok, tok), (h_msk, msk), (h_p, prompt),
-               (h_n, seqlen)]
-        outs = [(nt, o_tok), (nm, o_msk), (ne, o_ne)]
-        h2d = sum(h.numel() * h.element_size() for h, _ in ins)
-        d2h = sum(h.numel() * h.element_size() for _, h in outs)
-
-        def e2e_step():
-            for h, dv in ins:
-                dv.copy_(h, non_blocking=True)
-            step()
-            for dv, h in outs:
-                h.copy_(dv, non_blocking=True)
-
-        e2e_step()
-        torch.cuda.synchronize()
-        k_e2e = max(2, min(args.steps, 10))
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        e0.record(stream)
-        for _ in range(k_e2e):
-            e2e_step()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        te = max_over_ranks(e0.elapsed_time(e1) / k_e2e, world, d)
-        e2e = {"value": job_steps_per_s(te, world), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": te, "steps": k_e2e}
+    e2e = None if args.no_e2e else measure_e2e(args, Bn, w, bufs, stream, mask_mode, world, d,
+                                                  copy_streams=args.copy_streams)
 
     if rank != 0:
         return None
@@ -664,6 +714,7 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--copy-streams", type=int, default=4, help="host -> device copy streams of the end-to-end leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--loop-steps", type=int, default=4,
                     help="also time a recorded multi-pass loop with device-side early stop (0: skip)")
