@@ -12,16 +12,26 @@
  *   dlm_refine_update     commit masked positions, edit confident changes,
  *                         remask the k least confident positions
  *
- * dlm_refine_step does the last two in one launch (same results), and
- * dlm_loop_* repeat a recorded pass on the GPU until no confident edit remains.
+ * Around them:
+ *   dlm_refine_step          the last two in one launch (same results);
+ *                            dlm_refine_step_static without a workspace
+ *   dlm_lmhead_confidence    the vocabulary projection hidden x W^T fused with
+ *                            the per-position reduction (logits never stored)
+ *   dlm_attn_masked          block-causal / block-local attention (the
+ *                            block-autoregressive pattern and local refinement)
+ *   dlm_token_prob,          remask ranking by the probability of each
+ *   dlm_refine_update_ranked position's resulting token (a second reading)
+ *   dlm_loop_*               repeat a recorded pass on the GPU until no
+ *                            confident edit remains (one graph launch)
  *
  * Conventions shared by every call
  * --------------------------------
  * - Tensors are passed as dlm_tensor descriptors: a DEVICE pointer of the
  *   current CUDA device, a dtype, the shape and the strides in elements.
  *   The caller owns every buffer; the library allocates no device memory and
- *   keeps no pointer after a call returns. Its only device memory is static:
- *   the error word and the 16 KB scratch of dlm_refine_step_static.
+ *   keeps no pointer after a call returns (a dlm_loop keeps the pointers of
+ *   the calls it recorded). Its only device memory is static: the error word
+ *   and the 16 KB scratch of dlm_refine_step_static.
  * - Calls are asynchronous on the stream set by dlm_set_stream for the calling
  *   thread (default: the legacy default stream). Outputs are valid once that
  *   stream has been synchronised. Arguments are validated on the host before
@@ -43,7 +53,7 @@ extern "C" {
 #endif
 
 #define DLM_VERSION_MAJOR 0
-#define DLM_VERSION_MINOR 1
+#define DLM_VERSION_MINOR 2
 #define DLM_VERSION_PATCH 0
 
 typedef enum dlm_dtype {
