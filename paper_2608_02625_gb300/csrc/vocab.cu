@@ -8,7 +8,9 @@
 // An HBM-bound stream: every logit is read exactly once with 16-byte
 // non-allocating loads, coalesced across the block. Each thread keeps an
 // online (max, first index, scaled sum) triple; the sum is rescaled only when a
-// 16-byte vector raises the running maximum. Threads combine by warp shuffles,
+// 16-byte vector raises the running maximum, and the exponentials go two at a
+// time through the packed fp32 FMA and add of the sm_100 family, so that the
+// instruction stream stays below what HBM delivers per SM. Threads combine by warp shuffles,
 // warps through shared memory, and -- when there are too few rows to fill the
 // GPU -- the CTAs of a thread-block cluster that split one row combine through
 // distributed shared memory (no global scratch memory).
@@ -100,34 +102,45 @@ struct Vec<false> {
   }
 };
 
-// Folds one vector of kN values starting at element index e0 into p.
+// Folds one value x at element index e into p (the scalar path: rows whose
+// length or alignment rules out 16-byte vectors, and a row's ragged tail).
+__device__ __forceinline__ void fold1(Partial& p, float& mL, float x, int e) {
+  if (x > p.m) {
+    p.s = (p.m == -INFINITY) ? 0.f : p.s * ex2_approx((p.m - x) * kLog2e);
+    p.m = x;
+    p.idx = e;
+    mL = x * kLog2e;
+  }
+  if (p.m != -INFINITY) p.s += ex2_approx(fmaf(x, kLog2e, -mL));
+}
+
+// Folds one 16-byte vector of kN values starting at element index e0: the
+// vector's maximum first (raising the running maximum rescales the sum, which
+// is rare), then the kN exponentials in pairs with packed fp32 FMA and add
+// into the two-lane running sum s2. mL is the running maximum times log2(e)
+// and stays finite (0 until the first finite maximum): an entry of -inf then
+// adds exp2(-inf) = 0 without a guard.
 template <int kN>
-__device__ __forceinline__ void fold(Partial& p, float& mL, const float (&x)[kN], int e0) {
-  float vm = x[0];
-#pragma unroll
-  for (int j = 1; j < kN; ++j) vm = fmaxf(vm, x[j]);
+__device__ __forceinline__ void fold_vec(Partial& p, float& mL, float2& s2, const float (&x)[kN], int e0) {
+  float vm;
+  if constexpr (kN == 8) vm = fmaxf(fmax3(fmax3(x[0], x[1], x[2]), fmax3(x[3], x[4], x[5]), x[6]), x[7]);
+  else vm = fmaxf(fmax3(x[0], x[1], x[2]), x[3]);
   if (vm > p.m) {
     int first = kN - 1;
 #pragma unroll
     for (int j = kN - 1; j >= 0; --j)
       if (x[j] == vm) first = j;
-    p.s = (p.m == -INFINITY) ? 0.f : p.s * ex2_approx((p.m - vm) * kLog2e);
+    const float f = (p.m == -INFINITY) ? 0.f : ex2_approx((p.m - vm) * kLog2e);
+    s2 = make_float2(s2.x * f, s2.y * f);
     p.m = vm;
     p.idx = e0 + first;
     mL = vm * kLog2e;
   }
-  if (p.m != -INFINITY) {
-    if constexpr (kN == 1) {
-      p.s += ex2_approx(fmaf(x[0], kLog2e, -mL));
-    } else {
-      float a0 = 0.f, a1 = 0.f;
+  const float2 k2 = make_float2(kLog2e, kLog2e), n2 = make_float2(-mL, -mL);
 #pragma unroll
-      for (int j = 0; j < kN; j += 2) {
-        a0 += ex2_approx(fmaf(x[j], kLog2e, -mL));
-        a1 += ex2_approx(fmaf(x[j + 1], kLog2e, -mL));
-      }
-      p.s += a0 + a1;
-    }
+  for (int j = 0; j < kN; j += 2) {
+    const float2 y = ffma2(make_float2(x[j], x[j + 1]), k2, n2);
+    s2 = fadd2(s2, make_float2(ex2_approx(y.x), ex2_approx(y.y)));
   }
 }
 
@@ -171,6 +184,7 @@ __device__ __forceinline__ Partial scan_range(const char* row, int64_t e_begin, 
     const int64_t v_begin = e_begin / kN;
     const int64_t v_end = e_end / kN;  // full vectors
     const uint4* vp = reinterpret_cast<const uint4*>(row);
+    float2 s2 = make_float2(0.f, 0.f);
     int64_t vi = v_begin + threadIdx.x;
     for (; vi + (kUnroll - 1) * kThreads < v_end; vi += kUnroll * kThreads) {
       uint4 raw[kUnroll];
@@ -180,20 +194,19 @@ __device__ __forceinline__ Partial scan_range(const char* row, int64_t e_begin, 
       for (int u = 0; u < kUnroll; ++u) {
         float x[kN];
         VT::unpack(raw[u], x);
-        fold<kN>(p, mL, x, static_cast<int>((vi + u * kThreads) * kN));
+        fold_vec<kN>(p, mL, s2, x, static_cast<int>((vi + u * kThreads) * kN));
       }
     }
     for (; vi < v_end; vi += kThreads) {
       float x[kN];
       VT::unpack(ld_stream16(vp + vi), x);
-      fold<kN>(p, mL, x, static_cast<int>(vi * kN));
+      fold_vec<kN>(p, mL, s2, x, static_cast<int>(vi * kN));
     }
+    p.s = s2.x + s2.y;
     e_begin = v_end * kN;  // scalar tail (row length not a multiple of kN)
   }
-  for (int64_t e = e_begin + threadIdx.x; e < e_end; e += kThreads) {
-    float x[1] = {VT::load1(row, e)};
-    fold<1>(p, mL, x, static_cast<int>(e));
-  }
+  for (int64_t e = e_begin + threadIdx.x; e < e_end; e += kThreads)
+    fold1(p, mL, VT::load1(row, e), static_cast<int>(e));
   return p;
 }
 
