@@ -260,18 +260,22 @@ __global__ void __launch_bounds__(kThreads, 4) vocab_step_kernel(VocabArgs a, Up
   }
 }
 
-// A cluster of `csize` CTAs per row; CTA c scans a contiguous chunk, rank 0
-// combines the chunk partials through distributed shared memory.
+// Rows split over a cluster of `csize` CTAs: CTA c of a cluster scans chunk c
+// of the row, rank 0 combines the chunk partials through distributed shared
+// memory. Persistent: cluster k takes rows k, k + clusters, ..., so a launch is
+// one wave of resident CTAs, with no per-row launch and ramp-up; the partial
+// slots alternate between rows, so one cluster barrier per row suffices (rank
+// 0 reads row i's partials before it scans row i + 1, whose barrier the other
+// CTAs must pass before they overwrite that slot with row i + 2's).
 template <bool BF16, bool VEC>
 __global__ void __launch_bounds__(kThreads, 4) vocab_cluster_kernel(VocabArgs a) {
-  __shared__ Partial cta_part;
+  __shared__ Partial cta_part[2];
   cg::cluster_group cluster = cg::this_cluster();
   const int csize = static_cast<int>(cluster.num_blocks());
   const int crank = static_cast<int>(cluster.block_rank());
+  const int64_t nclusters = gridDim.x / csize;
   const int esz = BF16 ? 2 : 4;
   const int kN = BF16 ? 8 : 4;
-  const int64_t rowi = blockIdx.x / csize;
-  const char* row = static_cast<const char*>(a.logits) + rowi * a.row_stride * esz;
   // Chunk boundaries on whole vectors.
   const int64_t nvec = (a.V + kN - 1) / kN;
   const int64_t per = (nvec + csize - 1) / csize;
@@ -279,22 +283,26 @@ __global__ void __launch_bounds__(kThreads, 4) vocab_cluster_kernel(VocabArgs a)
   int64_t e1 = (crank + 1) * per * kN;
   if (e0 > a.V) e0 = a.V;
   if (e1 > a.V) e1 = a.V;
-  Partial p = scan_range<BF16, VEC>(row, e0, e1);
-  p = block_reduce(p);
-  if (threadIdx.x == 0) cta_part = p;
-  cluster.sync();
-  if (crank == 0 && threadIdx.x < 32) {
-    Partial q{-INFINITY, 0x7FFFFFFF, 0.f};
-    if (static_cast<int>(threadIdx.x) < csize) q = *cluster.map_shared_rank(&cta_part, threadIdx.x);
+  int it = 0;
+  for (int64_t rowi = blockIdx.x / csize; rowi < a.N; rowi += nclusters, ++it) {
+    const char* row = static_cast<const char*>(a.logits) + rowi * a.row_stride * esz;
+    Partial p = scan_range<BF16, VEC>(row, e0, e1);
+    p = block_reduce(p);
+    if (threadIdx.x == 0) cta_part[it & 1] = p;
+    cluster.sync();
+    if (crank == 0 && threadIdx.x < 32) {
+      Partial q{-INFINITY, 0x7FFFFFFF, 0.f};
+      if (static_cast<int>(threadIdx.x) < csize) q = *cluster.map_shared_rank(&cta_part[it & 1], threadIdx.x);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      Partial t;
-      t.m = __shfl_xor_sync(0xffffffffu, q.m, o);
-      t.idx = __shfl_xor_sync(0xffffffffu, q.idx, o);
-      t.s = __shfl_xor_sync(0xffffffffu, q.s, o);
-      q = combine(q, t);
+      for (int o = 16; o > 0; o >>= 1) {
+        Partial t;
+        t.m = __shfl_xor_sync(0xffffffffu, q.m, o);
+        t.idx = __shfl_xor_sync(0xffffffffu, q.idx, o);
+        t.s = __shfl_xor_sync(0xffffffffu, q.s, o);
+        q = combine(q, t);
+      }
+      if (threadIdx.x == 0) write_out(a, rowi, q);
     }
-    if (threadIdx.x == 0) write_out(a, rowi, q);
   }
   cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
 }
@@ -324,16 +332,32 @@ int launch_typed(const VocabArgs& a, cudaStream_t stream) {
   const int esz = BF16 ? 2 : 4;
   const int64_t row_bytes = a.V * esz;
   const int64_t want_ctas = 4LL * sms;  // resident CTAs at 4 per SM
-  int csize = 1;
-  if (row_bytes >= 65536) {
-    while (csize < 8 && a.N * csize < 2 * want_ctas) csize *= 2;
-  }
-  if (csize == 1) {
-    int64_t grid = a.N < 64LL * want_ctas ? a.N : 64LL * want_ctas;
+  // One CTA per row wherever there are rows enough to keep more than two CTAs
+  // per SM streaming: measured on this GPU (V = 151552, bf16), splitting rows
+  // over clusters wins only up to about 2 rows per SM (64 rows: 16 us against
+  // 21; 304: 22.6 against 24.9), and loses beyond (512 rows: 49.6 against 31.3,
+  // as each CTA's short chunks pay the memory latency once per row).
+  if (row_bytes < 65536 || a.N > 2LL * sms) {
+    const int64_t grid = a.N < 64LL * want_ctas ? a.N : 64LL * want_ctas;
     vocab_rows_kernel<BF16, VEC><<<static_cast<unsigned>(grid), kThreads, 0, stream>>>(a);
   } else {
+    // Few long rows: split each over a cluster. Choose the cluster size that
+    // minimises the rows' share per CTA, ceil(N / clusters) / csize, with
+    // clusters = resident CTAs / csize (never more clusters than rows).
+    int csize = 2;
+    int64_t nclusters = 1;
+    double best = 1e30;
+    for (int c = 2; c <= 8; c *= 2) {
+      int64_t nc = want_ctas / c;
+      if (nc > a.N) nc = a.N;
+      const double cost = static_cast<double>((a.N + nc - 1) / nc) / c;
+      if (cost < best - 1e-9) {
+        best = cost;
+        csize = c;
+        nclusters = nc;
+      }
+    }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(a.N * csize));
     cfg.blockDim = dim3(kThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -343,6 +367,15 @@ int launch_typed(const VocabArgs& a, cudaStream_t stream) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    // No more clusters than can be resident at once (one wave).
+    cfg.gridDim = dim3(static_cast<unsigned>(nclusters * csize));
+    int active = 0;
+    if (cudaOccupancyMaxActiveClusters(&active, vocab_cluster_kernel<BF16, VEC>, &cfg) == cudaSuccess && active > 0 &&
+        nclusters > active) {
+      nclusters = active;
+      cfg.gridDim = dim3(static_cast<unsigned>(nclusters * csize));
+    }
+    cudaGetLastError();  // an occupancy query that failed leaves the grid as computed
     cudaError_t e = cudaLaunchKernelEx(&cfg, vocab_cluster_kernel<BF16, VEC>, a);
     if (e != cudaSuccess)
       return fail(DLM_ERR_CUDA, "vocab_confidence cluster launch: %s", cudaGetErrorString(e));
