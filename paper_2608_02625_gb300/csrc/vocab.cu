@@ -216,6 +216,12 @@ __device__ __forceinline__ Partial scan_range(const char* row, int64_t e_begin, 
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
   asm volatile("cp.async.cg.shared.global.L2::256B [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
 }
+// The same copy, issued only once `after` holds its value: passing a register
+// loaded from the destination slot orders the slot's read before its refill.
+__device__ __forceinline__ void cp_async16_after(void* smem_dst, const void* gsrc, uint32_t after) {
+  asm volatile("cp.async.cg.shared.global.L2::256B [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc), "r"(after)
+               : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() {
@@ -225,8 +231,7 @@ __device__ __forceinline__ void cp_async_wait() {
 // scan_range for 16-byte aligned rows with the loads staged through shared
 // memory: each thread keeps kStages of its vectors in flight in its own slots
 // of `ring` ([kStages][kThreads]), reads back only what it copied itself (so
-// no block barrier), and refills a slot after the values read from it have
-// been used. Twice the bytes in flight of the register-loaded scan, with no
+// no block barrier), and refills a slot as soon as its value is in registers. Twice the bytes in flight of the register-loaded scan, with no
 // registers held for them.
 template <bool BF16, int kStages>
 __device__ __forceinline__ Partial scan_range_staged(const char* row, int64_t e_begin, int64_t e_end, uint4* ring) {
@@ -248,11 +253,12 @@ __device__ __forceinline__ Partial scan_range_staged(const char* row, int64_t e_
   for (int k = 0; k < nk; ++k) {
     cp_async_wait<kStages - 1>();  // the group of vector k has landed
     uint4* slot = mine + (k % kStages) * kThreads;
-    float x[kN];
-    VT::unpack(*slot, x);
-    fold_vec<kN>(p, mL, s2, x, static_cast<int>((first + static_cast<int64_t>(k) * kThreads) * kN));
-    if (k + kStages < nk) cp_async16(slot, vp + first + static_cast<int64_t>(k + kStages) * kThreads);
+    const uint4 v = *slot;
+    if (k + kStages < nk) cp_async16_after(slot, vp + first + static_cast<int64_t>(k + kStages) * kThreads, v.w);
     cp_async_commit();
+    float x[kN];
+    VT::unpack(v, x);
+    fold_vec<kN>(p, mL, s2, x, static_cast<int>((first + static_cast<int64_t>(k) * kThreads) * kN));
   }
   cp_async_wait<0>();
   p.s = s2.x + s2.y;

@@ -103,3 +103,15 @@ def test_strided_rows_and_3d():
     odd = wide[:, 3:3 + V]                   # rows not 16-byte aligned: scalar path
     ref_odd = oracle.vocab_confidence(odd.float().cpu().numpy())
     check_vocab(*gpu_vocab(odd), *ref_odd, where="unaligned")
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("N,V,pad", [(1000, 1003, 5), (2000, 64, 0), (700, 40000, 8), (900, 12, 4)])
+def test_many_rows_ragged(dtype, N, V, pad):
+    """More rows than one wave of resident CTAs (the staged scan), with row
+    lengths that leave a scalar tail, tiny rows (most threads idle) and padded
+    row strides."""
+    x = planted(N, V + pad, N + V)
+    t = to_dev(x, dtype)[:, :V]
+    ref = oracle.vocab_confidence(t.float().cpu().numpy())
+    check_vocab(*gpu_vocab(t), *ref, where=f"{dtype} {N}x{V}+{pad}")
