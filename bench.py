@@ -29,6 +29,15 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "refine_steps_per_sec"
+# The paper's own headline numbers (Table 1, Table 4): end-to-end seconds per
+# example of whole-model decoding on hardware it does not name. Context only:
+# they are speedups of a decoding scheme, not a refine-step throughput.
+PAPER_CONTEXT = {
+    "speedups": {"flash_flash_vs_selected_block_ar_gsm8k_384": 1.20, "mini_flash_vs_flash_math_384": 2.17},
+    "seconds_per_example": {"gsm8k_384": [19.38, 16.09], "math_384": [40.90, 18.82]},
+    "hardware": "not stated by the paper",
+    "comparable": False,
+}
 UNIT = "steps/s"
 DEFAULT_CONFIG = "c3_batch32_512"
 
@@ -671,6 +680,7 @@ def run_ours(args, rank, world):
         "e2e": e2e,
         "loop": loop_info,
         "lmhead": lmhead_info,
+        "paper_context": PAPER_CONTEXT,
     }
     if timer is not None:
         res["cpu_baseline"] = timer.run()
