@@ -92,12 +92,12 @@ def describe(t: torch.Tensor | None) -> DlmTensor | None:
     if t.dim() < 1 or t.dim() > 4:
         raise ValueError("tensors of rank 1..4 only")
     d = DlmTensor()
+    n = t.dim()
     d.data = t.data_ptr() if t.numel() else None
     d.dtype = _DTYPES[t.dtype]
-    d.ndim = t.dim()
-    for i in range(t.dim()):
-        d.shape[i] = t.shape[i]
-        d.stride[i] = t.stride(i)
+    d.ndim = n
+    d.shape[:n] = t.shape
+    d.stride[:n] = t.stride()
     return d
 
 
@@ -112,17 +112,21 @@ def _check(status: int):
 
 
 def _prepare(*tensors):
-    dev = None
+    dev = -1
     for t in tensors:
         if t is None:
             continue
-        if not t.is_cuda:
+        idx = t.get_device()
+        if idx < 0:
             raise ValueError("libdlmrefine takes CUDA tensors")
-        if dev is None:
-            dev = t.device
-        elif t.device != dev:
+        if dev < 0:
+            dev = idx
+        elif idx != dev:
             raise ValueError("all tensors must be on one device")
-    torch.cuda.set_device(dev)
+    if dev < 0:
+        raise ValueError("no tensor given")
+    if torch.cuda.current_device() != dev:
+        torch.cuda.set_device(dev)
     _check(lib.dlm_set_stream(ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)))
 
 
