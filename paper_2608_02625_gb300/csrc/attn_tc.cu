@@ -24,7 +24,8 @@
 //   warp 8     TMA producer: Q per unit and slot; K_0, K_1, V_0, K_2, V_1, K_3, ...
 //              through a ring of eight sub-tile slots, each released as soon as
 //              the MMAs that read it have completed
-//   warp 9     tensor-memory allocator; MMA issuer of slot 0 (one elected thread)
+//   warp 9     tensor-memory allocator; MMA issuer of slot 0 (one lane elected
+//              per instruction)
 //   warp 10    MMA issuer of slot 1
 // Tensor memory (512 columns x 128 lanes x 32 bit), slot i at column 256 i:
 //   S_i buffers 0 and 1   fp32 128 x 64 at +0 and +64 (sub-tile j uses buffer j % 2)
@@ -322,13 +323,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp >= kMmaWarp0) {
     // ================================================================ MMA issuers
-    // Warp kMmaWarp0 + i issues every MMA of slot i (one elected thread), so the
-    // two slots' MMA streams do not wait on each other's hand-offs; each
-    // stream is ordered on its own. Both issuers arrive on every ring slot's
-    // release barrier: with tcgen05.commit after their MMAs read the slot, or
-    // with a plain arrive (after the fill landed) when their slot idles in a unit.
+    // Warp kMmaWarp0 + i issues every MMA of slot i, so the two slots' MMA
+    // streams do not wait on each other's hand-offs; each stream is ordered on
+    // its own. All 32 lanes run the issue loop (waits are warp-uniform) and
+    // one lane elected inside each instruction issues it: no branch around the
+    // MMAs, whose operands then stay in uniform registers. Both issuers arrive
+    // on every ring slot's release barrier: with tcgen05.commit after their
+    // MMAs read the slot, or with a plain arrive (after the fill landed) when
+    // their slot idles in a unit.
     const int i = warp - kMmaWarp0;
-    if (lane == 0) {
+    {
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, kSub, false, false);  // Q, K both K-major
       constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);      // V is MN-major (D contiguous)
       const uint32_t q_addr = smem_u32(sm.q[i]);
@@ -340,10 +344,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t qoff = (kk / 4) * kQBoxBytes + (kk % 4) * 32;
           const uint32_t koff = (kk / 4) * kKvBoxBytes + (kk % 4) * 32;
-          mma_ss(s_tmem + kSub * b, sdesc_sw128(q_addr + qoff, 16, 1024), sdesc_sw128(kaddr + koff, 16, 1024),
+          mma_ss_elect(s_tmem + kSub * b, sdesc_sw128(q_addr + qoff, 16, 1024), sdesc_sw128(kaddr + koff, 16, 1024),
                  idesc_s, kk > 0);
         }
-        mma_commit(&sm.bar_s[i][b]);
+        mma_commit_elect(&sm.bar_s[i][b]);
       };
       // O_i (+)= P_i(j) [128 x 64, tensor memory] times V sub-tile [64 x D].
       // Only the unit's last two PVs signal their completion (bar_pvm, bar_o):
@@ -352,17 +356,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t vaddr = smem_u32(sm.ring[r]);
 #pragma unroll
         for (int kk = 0; kk < kSub / 16; ++kk) {
-          mma_ts(s_tmem + 128, s_tmem + kSub * b + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kKvBoxBytes, 1024),
+          mma_ts_elect(s_tmem + 128, s_tmem + kSub * b + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kKvBoxBytes, 1024),
                  idesc_o, (acc || kk > 0) ? 1u : 0u);
         }
-        if (done) mma_commit(done);
+        if (done) mma_commit_elect(done);
       };
       auto wait_fill = [&](int f) -> bool {
-        return mbar_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err);
+        return warp_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err);
       };
       auto release = [&](int f, bool issued) {
-        if (issued) mma_commit(&sm.bar_empty[f % kRing]);
-        else mbar_arrive(&sm.bar_empty[f % kRing]);
+        if (issued) mma_commit_elect(&sm.bar_empty[f % kRing]);
+        else mbar_arrive_elect(&sm.bar_empty[f % kRing]);
       };
       int q_loads = 0;    // bar_q phases consumed
       int units_run = 0;  // bar_ofree phases
@@ -374,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (U.nkv == 0) continue;
         const bool run = U.run[i];
         if (run) {
-          ok = mbar_wait(&sm.bar_q[i], q_loads & 1, abort, p.err);
+          ok = warp_wait(&sm.bar_q[i], q_loads & 1, abort, p.err);
           ++q_loads;
         }
         // Prologue: S(0) and S(1) into buffers 0 and 1.
@@ -383,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (run) {
             tc_fence_after();
             issue_s(j, f % kRing);
-            if (j == U.nkv - 1) mma_commit(&sm.bar_qfree[i]);
+            if (j == U.nkv - 1) mma_commit_elect(&sm.bar_qfree[i]);
           }
           release(f, run);
         }
@@ -392,11 +396,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!wait_fill(fv)) { ok = false; break; }
           if (run) {
             // O_i of this slot's previous unit must have been read out before PV(0) overwrites it.
-            if (j == 0 && units_run > 0 && !mbar_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err)) {
+            if (j == 0 && units_run > 0 && !warp_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err)) {
               ok = false;
               break;
             }
-            if (!mbar_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
+            if (!warp_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
             ++p_seen;
             tc_fence_after();
             issue_pv(j & 1, fv % kRing, j > 0,
@@ -409,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (run) {
               tc_fence_after();
               issue_s(j & 1, fk % kRing);
-              if (j + 2 == U.nkv - 1) mma_commit(&sm.bar_qfree[i]);
+              if (j + 2 == U.nkv - 1) mma_commit_elect(&sm.bar_qfree[i]);
             }
             release(fk, run);
           }
@@ -417,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (run) ++units_run;
       }
       // Teardown: every MMA issued by this thread completes before TMEM is freed.
-      mma_commit(&sm.bar_done[i]);
+      mma_commit_elect(&sm.bar_done[i]);
       mbar_drain(&sm.bar_done[i], 0);
     }
     __syncwarp();
