@@ -155,7 +155,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 1) {
     // ================================================================ MMA issuer
-    if (lane == 0) {
+    // All 32 lanes run the loop (warp-uniform waits); one lane elected inside
+    // each MMA / commit issues it, with no branch around the MMAs.
+    {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, false, false);  // both operands K-major
       int fill = 0, tile = 0;
       bool ok = true;
@@ -164,7 +166,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int vt = it.t0; ok && vt < it.t1; ++vt, ++tile) {
           const int acc = tile & 1;
           // The accumulator's previous tile (tile - 2) must have been read out.
-          if (tile >= 2 && !mbar_wait(&sm.acc_empty[acc], ((tile >> 1) - 1) & 1, abort, p.err)) {
+          if (tile >= 2 && !warp_wait(&sm.acc_empty[acc], ((tile >> 1) - 1) & 1, abort, p.err)) {
             ok = false;
             break;
           }
@@ -172,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t d_tmem = tmem + acc * kBN;
           for (int kb = 0; kb < kblocks; ++kb, ++fill) {
             const int st = fill % kStages;
-            if (!mbar_wait(&sm.full[st], (fill / kStages) & 1, abort, p.err)) {
+            if (!warp_wait(&sm.full[st], (fill / kStages) & 1, abort, p.err)) {
               ok = false;
               break;
             }
@@ -181,15 +183,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t b_addr = smem_u32(sm.b[st]);
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-              mma_ss(d_tmem, sdesc_sw128(a_addr + kk * 32, 16, 1024), sdesc_sw128(b_addr + kk * 32, 16, 1024), idesc,
-                     (kb > 0 || kk > 0) ? 1u : 0u);
-            mma_commit(&sm.empty[st]);
+              mma_ss_elect(d_tmem, sdesc_sw128(a_addr + kk * 32, 16, 1024), sdesc_sw128(b_addr + kk * 32, 16, 1024),
+                           idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            mma_commit_elect(&sm.empty[st]);
           }
           if (!ok) break;
-          mma_commit(&sm.acc_full[acc]);
+          mma_commit_elect(&sm.acc_full[acc]);
         }
       }
-      mma_commit(&sm.done);
+      mma_commit_elect(&sm.done);
       mbar_drain(&sm.done, 0);
     }
     __syncwarp();
