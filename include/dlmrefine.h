@@ -54,7 +54,7 @@ extern "C" {
 
 #define DLM_VERSION_MAJOR 0
 #define DLM_VERSION_MINOR 2
-#define DLM_VERSION_PATCH 0
+#define DLM_VERSION_PATCH 1
 
 typedef enum dlm_dtype {
   DLM_BF16 = 1, /* bfloat16 */
@@ -80,6 +80,12 @@ typedef enum dlm_status {
 #define DLM_DEVERR_LENGTH 0x1   /* a seq_len / prompt_len outside [0, L] was clamped */
 #define DLM_DEVERR_TIMEOUT 0x2  /* a bounded wait in a kernel gave up; its outputs are undefined */
 #define DLM_DEVERR_NAN 0x4      /* a NaN confidence reached the remask selection */
+/* An input outside its contract was seen: a row of logits with a NaN entry or
+ * with every entry -inf (dlm_vocab_confidence, dlm_refine_step), a token id
+ * outside [0, V) (dlm_token_prob). Checked only by builds compiled with
+ * DLM_CHECK_BOUNDS (python -m paper_2608_02625_gb300.build --check-bounds);
+ * the default build leaves such outputs undefined, as documented per call. */
+#define DLM_DEVERR_INPUT 0x8
 
 typedef struct dlm_tensor {
   void* data;        /* device pointer; 16-byte aligned where a call requires it */

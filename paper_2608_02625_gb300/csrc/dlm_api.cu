@@ -306,6 +306,7 @@ int prepare_logits(const dlm_tensor* logits, dlm::VocabArgs* a) {
   a->N = N;
   a->V = V;
   a->row_stride = N > 1 ? row_stride : V;
+  a->err = dlm::device_error_word();
   return DLM_OK;
 }
 

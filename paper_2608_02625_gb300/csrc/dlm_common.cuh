@@ -341,6 +341,15 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N, bo
          ((b_mn_major ? 1u : 0u) << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
+// Builds compiled with DLM_CHECK_BOUNDS check the inputs' value contracts in
+// the kernels (NaN or all -inf logit rows, token ids out of range) and report
+// a violation as DLM_DEVERR_INPUT; the default build does not pay for it.
+#ifdef DLM_CHECK_BOUNDS
+constexpr bool kCheckBounds = true;
+#else
+constexpr bool kCheckBounds = false;
+#endif
+
 // ----------------------------------------------------------------- math
 
 __device__ __forceinline__ float ex2_approx(float x) {

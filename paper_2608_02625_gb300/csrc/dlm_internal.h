@@ -42,6 +42,7 @@ struct VocabArgs {
   int32_t* argmax;
   float* conf;
   float* lse;
+  int* err;  // device error word (input checks of DLM_CHECK_BOUNDS builds)
 };
 
 int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream);

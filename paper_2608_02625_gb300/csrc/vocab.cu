@@ -268,6 +268,8 @@ __device__ __forceinline__ Partial scan_range_staged(const char* row, int64_t e_
 }
 
 __device__ __forceinline__ void write_out(const VocabArgs& a, int64_t rowi, Partial p) {
+  // A NaN entry makes the sum NaN; a row of only -inf leaves the maximum -inf.
+  if (kCheckBounds && (isnan(p.s) || p.m == -INFINITY)) set_device_error(a.err, DLM_DEVERR_INPUT);
   a.argmax[rowi] = p.idx;
   a.conf[rowi] = 1.0f / p.s;
   a.lse[rowi] = p.m + logf(p.s);
@@ -376,6 +378,7 @@ __global__ void __launch_bounds__(256) token_prob_kernel(VocabArgs a, const int3
   if (r >= a.N) return;
   const int32_t t = tokens[r];
   float p = 0.f;
+  if (kCheckBounds && (t < 0 || t >= a.V)) set_device_error(a.err, DLM_DEVERR_INPUT);
   if (t >= 0 && t < a.V) {
     const int64_t off = r * a.row_stride + t;
     const float x = BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(a.logits)[off])

@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(header, lib):
 
 def test_version_and_status_strings():
     from paper_2608_02625_gb300 import binding as B
-    assert B.dlm_version() == 200
+    assert B.dlm_version() == 201
     assert B.dlm_status_string(0) == "ok"
     assert "dtype" in B.dlm_status_string(-2)
 
