@@ -115,3 +115,19 @@ def test_many_rows_ragged(dtype, N, V, pad):
     t = to_dev(x, dtype)[:, :V]
     ref = oracle.vocab_confidence(t.float().cpu().numpy())
     check_vocab(*gpu_vocab(t), *ref, where=f"{dtype} {N}x{V}+{pad}")
+
+
+@pytest.mark.parametrize("dtype,N,V", [("bf16", 200, 151552), ("f32", 160, 65536), ("bf16", 100, 151552)])
+def test_split_rows_several_per_cluster(dtype, N, V):
+    """Few long rows (at most two per SM): each row is split over a cluster, and
+    with these counts a cluster takes several rows in turn (alternating partial
+    slots); ties planted across the chunk boundaries of a cluster."""
+    x = planted(N, V, N + V + 1)
+    chunk = V // 8
+    for r in range(0, N, 7):
+        x[r, [chunk - 1, 3 * chunk + 5, V - 1]] = 30.0   # equal maxima in different CTAs' chunks
+    t = to_dev(x, dtype)
+    am, cf, ls = gpu_vocab(t)
+    ref = oracle.vocab_confidence(t.float().cpu().numpy())
+    check_vocab(am, cf, ls, *ref, where=f"{dtype} {N}x{V}")
+    assert all(am[r] == chunk - 1 for r in range(0, N, 7))
