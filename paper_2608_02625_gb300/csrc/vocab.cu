@@ -8,14 +8,14 @@
 // An HBM-bound stream: every logit is read exactly once, 16 bytes per load,
 // coalesced across the block; with several waves of rows the loads go through
 // a per-thread shared-memory staging ring (cp.async, eight vectors in flight
-// per thread), otherwise straight into registers (four in flight). Each thread keeps an
-// online (max, first index, scaled sum) triple; the sum is rescaled only when a
-// 16-byte vector raises the running maximum, and the exponentials go two at a
-// time through the packed fp32 FMA and add of the sm_100 family, so that the
-// instruction stream stays below what HBM delivers per SM. Threads combine by warp shuffles,
-// warps through shared memory, and -- when there are too few rows to fill the
-// GPU -- the CTAs of a thread-block cluster that split one row combine through
-// distributed shared memory (no global scratch memory).
+// per thread), otherwise straight into registers (four in flight). Each thread
+// keeps an online (max, first index, scaled sum) triple; the sum is rescaled
+// only when a 16-byte vector raises the running maximum, and the exponentials
+// go two at a time through the packed fp32 FMA and add of the sm_100 family,
+// so that the instruction stream stays below what HBM delivers per SM.
+// Threads combine by warp shuffles, warps through shared memory, and -- with
+// at most two rows per SM -- the CTAs of a thread-block cluster that split one
+// row combine through distributed shared memory (no global scratch memory).
 //
 // The fused variant (vocab_step_kernel) also runs step A3: the CTA finishing a
 // sequence's last row performs its update, counted with one int32 arrival
@@ -231,8 +231,9 @@ __device__ __forceinline__ void cp_async_wait() {
 // scan_range for 16-byte aligned rows with the loads staged through shared
 // memory: each thread keeps kStages of its vectors in flight in its own slots
 // of `ring` ([kStages][kThreads]), reads back only what it copied itself (so
-// no block barrier), and refills a slot as soon as its value is in registers. Twice the bytes in flight of the register-loaded scan, with no
-// registers held for them.
+// no block barrier), and refills a slot as soon as its value is in registers:
+// twice the bytes in flight of the register-loaded scan, with no registers
+// held for them.
 template <bool BF16, int kStages>
 __device__ __forceinline__ Partial scan_range_staged(const char* row, int64_t e_begin, int64_t e_end, uint4* ring) {
   using VT = Vec<BF16>;
