@@ -13,7 +13,8 @@
 // tile:
 //   warp 0     TMA producer: hidden box 128 x 64 and weight box 256 x 64 per
 //              64-wide K step, through a 4-stage ring (48 KB a stage)
-//   warp 1     tensor-memory allocator and MMA issuer (one elected thread):
+//   warp 1     tensor-memory allocator and MMA issuer (all lanes run the loop,
+//              one lane elected per instruction):
 //              tcgen05.mma kind::f16, M = 128, N = 256, K = 16, bf16 x bf16 ->
 //              fp32 accumulators; two accumulators of 256 columns, so the
 //              epilogue of a tile overlaps the K loop of the next
