@@ -206,7 +206,9 @@ class OracleTimer:
             self.procs.append(pr)
         self.ready = False
 
-    def _wait_ready(self):
+    def wait_ready(self):
+        """Block until every worker has generated its inputs (they use the host
+        cores and memory bandwidth until then)."""
         if not self.ready:
             for c in self.conns:
                 assert c.recv() == "ready"
@@ -214,7 +216,7 @@ class OracleTimer:
 
     def run(self):
         """One round: every worker times its sequence. Returns cpu_baseline."""
-        self._wait_ready()
+        self.wait_ready()
         for c in self.conns:
             c.send("run")
         parts = [c.recv() for c in self.conns]
@@ -582,6 +584,10 @@ def run_ours(args, rank, world):
     step = build_step(Bn, w, bufs, args, stream, mask_mode)
     out, params = bufs["out"], bufs["params"]
 
+    if timer is not None:
+        # The workers' input generation would compete with the host-link copies
+        # of the end-to-end leg: let it finish before anything is timed.
+        timer.wait_ready()
     clk = ClockSampler(d.index if d.index is not None else 0).__enter__()
     for _ in range(args.warmup):
         step()
