@@ -527,7 +527,11 @@ def measure_e2e(args, Bn, w, bufs, stream, mask_mode, world, d, copy_streams=4):
             if s + 1 < nsteps:
                 pending = nxt
 
-    run(2)
+    # Warm-up: after the host link has idled, host -> device copies start slow
+    # and reach their full rate only after ~0.3 s of traffic (measured on this
+    # GPU: 18, 57, then 212 GB/s over the first three 4 GB copies after 2 s of
+    # idling), so the leg runs 20 untimed steps (~0.5 s of copies) first.
+    run(20)
     torch.cuda.synchronize()
     k_e2e = max(4, min(args.steps, 20))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
