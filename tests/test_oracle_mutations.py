@@ -49,6 +49,8 @@ MUTATIONS = {
 }
 
 
+# A planted mask slip can leave a query row with no keys (a NaN row): expected.
+@pytest.mark.filterwarnings("ignore:invalid value encountered:RuntimeWarning")
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
 def test_mutation_is_caught(name, monkeypatch):
     mod, attr, fn, pins = MUTATIONS[name]
