@@ -10,8 +10,12 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_peaks_are_the_measured_ones():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     pk = bench.load_peaks()
-    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+    if not os.path.exists(path):  # written per machine, not committed
+        assert pk["source"] == "fallback"
+        return
+    with open(path) as f:
         m = json.load(f)
     assert pk["source"] == "measured"
     assert pk["hbm_gbs"] == m["hbm_gbs"] and pk["bf16_tflops"] == m["bf16_tflops"]
