@@ -185,7 +185,8 @@ def _oracle_worker(conn, name, b, vocab_rows):
 
 
 class OracleTimer:
-    """`workers` single-threaded processes (spawned), one sequence each."""
+    """Single-threaded processes (spawned, at most one per sequence of the
+    batch), each timing one sequence."""
 
     VOCAB_ROWS = 64
 
@@ -193,6 +194,8 @@ class OracleTimer:
         from paper_2608_02625_gb300 import workloads
         self.w = workloads.get(name)
         self.name = name
+        # No more workers than sequences: a step has B sequences to spread.
+        workers = max(1, min(workers, self.w.B))
         os.environ["OPENBLAS_NUM_THREADS"] = "1"
         os.environ["OMP_NUM_THREADS"] = "1"
         ctx = mp.get_context("spawn")

@@ -64,3 +64,21 @@ def test_source_sha_covers_the_shared_headers(monkeypatch):
     monkeypatch.setattr("builtins.open", spy)
     bench.kernel_source_sha("attn_tc.cu")
     assert {"attn_tc.cu", "dlm_common.cuh", "update_impl.cuh"} <= set(seen)
+
+
+def test_reference_arm_json_line():
+    """bench.py --impl reference on the tiny workload: one JSON line with the
+    contract's keys; the oracle's workers never outnumber the sequences."""
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config",
+                        "c1_tiny_f32", "--steps", "1", "--warmup", "3"], capture_output=True, text=True, timeout=300,
+                       cwd=ROOT)
+    assert r.returncode == 0, r.stderr
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    assert d["impl"] == "reference" and d["metric"] == "refine_steps_per_sec" and d["unit"] == "steps/s"
+    assert d["higher_is_better"] is True and d["value"] > 0
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] == 1  # c1 has one sequence
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert d["config"]["workload"] == "c1_tiny_f32"
