@@ -22,6 +22,11 @@ which any response position may be revised. One pass on the hot path is
   optionally ranked by the probability of each position's resulting token,
   with ``vocab.token_prob`` giving the probability of a kept token.
 
+``loop.refine_passes`` repeats such passes over a batch, each on the state the
+last one left, until a pass makes no confident edit or a pass budget is spent
+(Sec. 4.2's T_r passes; Appendix C.4's early stop when no confident edits
+remain).
+
 ``lmhead.lm_head_confidence`` is the vocabulary projection (hidden states times
 the output weights) followed by ``vocab.vocab_confidence``, the operation of
 the fused projection + reduction kernel.
@@ -37,3 +42,4 @@ from .attention import bidir_attn  # noqa: F401
 from .vocab import token_prob, vocab_confidence  # noqa: F401
 from .update import refine_update, remask_count  # noqa: F401
 from .lmhead import lm_head_confidence, lm_head_logits  # noqa: F401
+from .loop import refine_passes  # noqa: F401

@@ -537,4 +537,103 @@ def pin_update_result_ranking():
 UPDATE_PINS = [pin_update_golden, pin_update_invariants, pin_update_rank_count,
                pin_update_remask_fraction, pin_update_result_ranking]
 
-ALL_PINS = ATTN_PINS + VOCAB_PINS + UPDATE_PINS
+
+# ---------------------------------------------------------------- multi-pass loop
+
+def loop_golden_cases():
+    with open(os.path.join(GOLDEN, "loop_hand_examples.json")) as f:
+        return json.load(f)["cases"]
+
+
+def run_loop_case(c, max_passes=None):
+    logits = np.log(np.array(c["probs"], dtype=np.float64))   # [pass, B, L, V]
+
+    def logits_for(tok, msk, t):
+        return logits[min(t, len(logits) - 1)].reshape(-1, c["V"])
+
+    return oracle.refine_passes(np.array(c["tokens"]), np.array(c["mask"]), logits_for,
+                                max_passes=c["max_passes"] if max_passes is None else max_passes,
+                                edit_threshold=c["edit_threshold"], remask_k=c["remask_k"],
+                                remask_frac=c["remask_frac"], mask_id=c["mask_id"],
+                                prompt_lens=c["prompt_lens"], seq_lens=c["seq_lens"])
+
+
+def pin_loop_golden():
+    """Hand-worked passes (tests/golden/loop_hand_examples.json): a batch-level
+    stop after the first pass without a confident edit, and pass budgets."""
+    for c in loop_golden_cases():
+        r = run_loop_case(c)
+        assert r["passes"] == c["expect_passes"], c["name"]
+        assert r["tokens"].tolist() == c["expect_tokens"], c["name"]
+        assert r["mask"].tolist() == c["expect_mask"], c["name"]
+        assert r["n_edits"].tolist() == c["expect_n_edits"], c["name"]
+
+
+def _loop_state(rng, B=3, L=24, V=16):
+    p = rng.integers(0, L // 3, B)
+    n = np.minimum(L, p + rng.integers(1, L, B))
+    tok = rng.integers(0, V, (B, L)).astype(np.int32)
+    msk = (rng.random((B, L)) < 0.3).astype(np.uint8)
+    tok[msk == 1] = V
+    return tok, msk, p, n
+
+
+def pin_loop_unreachable_threshold():
+    """A threshold above 1 admits no edit (a confidence is at most 1): one
+    pass, whatever the budget, equal to one refine_update."""
+    rng = np.random.default_rng(41)
+    for trial in range(10):
+        tok, msk, p, n = _loop_state(rng)
+        x = rng.standard_normal((tok.size, 16)) * 3
+        for budget in (1, 2, 7):
+            r = oracle.refine_passes(tok, msk, lambda t, m, i: x, max_passes=budget, edit_threshold=1.5,
+                                     remask_k=2, remask_frac=0.0, mask_id=16, prompt_lens=p, seq_lens=n)
+            assert r["passes"] == 1 and not r["n_edits"].any()
+
+
+def pin_loop_commits_only_stop():
+    """Masked positions committed but every filled prediction equal to its
+    token: commits are not edits, so the first pass is the last."""
+    rng = np.random.default_rng(42)
+    tok, msk, p, n = _loop_state(rng)
+    V = 16
+    pred = np.where(msk == 1, rng.integers(0, V, tok.shape), tok)
+    x = np.full((tok.size, V), -5.0)
+    x[np.arange(tok.size), pred.reshape(-1)] = 5.0
+    r = oracle.refine_passes(tok, msk, lambda t, m, i: x, max_passes=9, edit_threshold=0.5, remask_k=0,
+                             remask_frac=0.0, mask_id=V, prompt_lens=p, seq_lens=n)
+    assert r["passes"] == 1
+    for b in range(tok.shape[0]):
+        resp = np.arange(p[b], n[b])
+        assert np.array_equal(r["tokens"][b, resp], pred[b, resp])     # every masked position committed
+        assert not r["mask"][b, resp].any()
+
+
+def pin_loop_budget():
+    """Predictions that flip every pass between two tokens with probability
+    ~0.9 edit every filled response position every pass: the loop runs exactly
+    max_passes passes, and the final tokens follow the parity of the count."""
+    B, L, V = 2, 10, 8
+    p, n = np.array([3, 0]), np.array([10, 7])
+    tok = np.zeros((B, L), dtype=np.int32)
+    msk = np.zeros((B, L), dtype=np.uint8)
+
+    def logits_for(t, m, i):
+        x = np.full((B * L, V), -3.0)
+        x[:, 1 if i % 2 == 0 else 0] = 3.0   # pass 0 predicts 1, pass 1 predicts 0, ...
+        return x
+
+    for budget in range(1, 6):
+        r = oracle.refine_passes(tok, msk, logits_for, max_passes=budget, edit_threshold=0.8, remask_k=0,
+                                 remask_frac=0.0, mask_id=V, prompt_lens=p, seq_lens=n)
+        assert r["passes"] == budget
+        want = 1 if budget % 2 == 1 else 0
+        for b in range(B):
+            assert np.all(r["tokens"][b, p[b]:n[b]] == want)
+            assert np.all(r["tokens"][b, :p[b]] == 0) and np.all(r["tokens"][b, n[b]:] == 0)
+        assert np.all(r["n_edits"] == n - p)
+
+
+LOOP_PINS = [pin_loop_golden, pin_loop_unreachable_threshold, pin_loop_commits_only_stop, pin_loop_budget]
+
+ALL_PINS = ATTN_PINS + VOCAB_PINS + UPDATE_PINS + LOOP_PINS

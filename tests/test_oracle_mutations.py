@@ -6,8 +6,10 @@ last instead of the first maximum, a strict threshold, ties broken towards the
 higher index, a rounded-up remask count, a block-causal mask that drops the
 query's own block, a block-local mask without the prompt, a resulting-token ranking that
 ignores which positions end with their argmax, a sign slip in a token's
-probability, a projection that pairs the wrong feature indices. If a pin suite let one through, the
-oracle could carry that slip undetected."""
+probability, a projection that pairs the wrong feature indices, and in the
+multi-pass loop: a budget off by one, a stop as soon as one sequence makes no
+edit, commits counted as edits, a stop rule that ignores the edits. If a pin
+suite let one through, the oracle could carry that slip undetected."""
 import math
 
 import numpy as np
@@ -18,6 +20,7 @@ from oracle import attention as oatt
 from oracle import update as oupd
 from oracle import lmhead as olmh
 from oracle import vocab as ovoc
+from oracle import loop as oloop
 
 MUTATIONS = {
     "causal_mask": (oatt, "key_mask", lambda n, p=0, block=1, mode=0: np.tril(np.ones((n, n), dtype=bool)),
@@ -42,6 +45,15 @@ MUTATIONS = {
     "result_rank_ignores_argmax": (oupd, "resulting_token_prob", lambda nt, pred, c, tp: tp, P.UPDATE_PINS),
     "token_prob_sign": (ovoc, "softmax_prob", lambda x, lse: float(np.exp(lse - x)), P.VOCAB_PINS),
     "projection_reversed_features": (olmh, "project", lambda h, w: h @ w[:, ::-1].T, P.VOCAB_PINS),
+    "loop_budget_plus_one": (oloop, "more_passes", lambda ne, passes, mx: passes <= mx and bool(np.any(ne > 0)),
+                             P.LOOP_PINS),
+    "loop_stops_per_sequence": (oloop, "more_passes", lambda ne, passes, mx: passes < mx and bool(np.all(ne > 0)),
+                                P.LOOP_PINS),
+    "loop_ignores_edits": (oloop, "more_passes", lambda ne, passes, mx: passes < mx, P.LOOP_PINS),
+    "loop_counts_commits": (oloop, "refine_update",
+                            lambda tok, msk, am, cf, **kw: (lambda r: (r[0], r[1], r[2] + np.asarray(msk).sum(
+                                axis=1).astype(np.int32)))(oupd.refine_update(tok, msk, am, cf, **kw)),
+                            P.LOOP_PINS),
     "ceil_remask_count": (oupd, "remask_count",
                           lambda k, f, r: max(0, min(k if k >= 0 else
                                                      math.ceil(float(np.float32(f)) * r), r)),
