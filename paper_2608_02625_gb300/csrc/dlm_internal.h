@@ -12,6 +12,10 @@ namespace dlm {
 // Device address of the error word of the current device (set up once per device).
 int* device_error_word();
 
+// Device address of dlm_refine_step_static's scratch array on the current
+// device (set up on first use; a status, with *out untouched, on failure).
+int static_step_scratch(int32_t** out);
+
 // Records a failure message for dlm_last_error() and returns `status`.
 int fail(int status, const char* fmt, ...);
 // Clears the calling thread's failure message (at the start of every entry point).
@@ -46,6 +50,14 @@ struct VocabArgs {
 };
 
 int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream);
+
+// The same reduction with a caller workspace of vocab_workspace_bytes(N)
+// bytes (zero on entry, left zero): with few rows, the logits are split
+// evenly over all CTAs and each row's partials merged through the workspace.
+constexpr int kVocabFlatMaxCtas = 4096;
+constexpr int kVocabFlatMaxRowsPerCta = 8;
+size_t vocab_workspace_bytes(int64_t N);
+int launch_vocab_confidence_ws(const VocabArgs& a, void* workspace, cudaStream_t stream);
 
 struct UpdateArgs {
   const int32_t* tokens;

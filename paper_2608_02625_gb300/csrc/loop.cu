@@ -19,9 +19,15 @@ constexpr int kCondThreads = 256;
 
 __global__ void loop_init_kernel(int32_t* steps) { *steps = 0; }
 
+// Error-word bits that end the loop: a bounded wait that gave up, a NaN
+// confidence, an input outside its contract -- the pass's outputs are then
+// undefined. A clamped sequence or prompt length (DLM_DEVERR_LENGTH) does
+// not: the kernels define the clamped result, so the pass is valid.
+constexpr int kStopBits = ~DLM_DEVERR_LENGTH;
+
 // Ends one pass: steps += 1; run another pass iff steps < max_steps, some
-// sequence had an edit (n_edits[b] > 0) and no kernel has set the device
-// error word.
+// sequence had an edit (n_edits[b] > 0) and no kernel has set a bit of
+// kStopBits in the device error word.
 __global__ void __launch_bounds__(kCondThreads)
     loop_cond_kernel(cudaGraphConditionalHandle handle, const int32_t* n_edits, int64_t batch, int32_t max_steps,
                      int32_t* steps, const int* err) {
@@ -36,7 +42,7 @@ __global__ void __launch_bounds__(kCondThreads)
     for (int w = 0; w < kCondThreads / 32; ++w) edits |= any_warp[w];
     const int n = *steps + 1;
     *steps = n;
-    const bool failed = *reinterpret_cast<const volatile int*>(err) != 0;
+    const bool failed = (*reinterpret_cast<const volatile int*>(err) & kStopBits) != 0;
     cudaGraphSetConditional(handle, (n < max_steps && edits && !failed) ? 1u : 0u);
   }
 }
@@ -72,8 +78,11 @@ int dlm_loop_begin(int32_t* steps_out) {
   cudaError_t e = cudaStreamIsCapturing(stream, &cs);
   if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "cudaStreamIsCapturing: %s", cudaGetErrorString(e));
   if (cs != cudaStreamCaptureStatusNone) return fail(DLM_ERR_ARG, "the stream is already capturing");
-  // Set-up that must not happen during the capture.
+  // Set-up that must not happen during the capture: the device addresses of
+  // the error word and of the static step scratch (cudaGetSymbolAddress).
   if (!dlm::device_error_word()) return fail(DLM_ERR_CUDA, "device error word unavailable");
+  int32_t* scratch = nullptr;
+  if (const int st = dlm::static_step_scratch(&scratch)) return st;
 
   cudaGraph_t g = nullptr;
   if ((e = cudaGraphCreate(&g, 0)) != cudaSuccess)

@@ -18,13 +18,30 @@ from oracle import remask_count
 # terms each with an exp2 of relative error ~2^-22).
 ATTN_TOL_BF16 = 2e-2
 ATTN_TOL_F32 = 1e-5
-# Peaked attention (q, k, v ~ N(0, 1) or wider): the bf16 output alone rounds
-# by up to 2^-9 |out| and the bf16 softmax numerators by 2^-9 max|v|, so the
-# absolute bound grows with the magnitude of v; these cases use
-# 2e-2 + 1e-2 * |ref|.
-ATTN_RTOL_PEAKED = 1e-2
+# Bounds scaled to the output, which a small systematic error would break
+# even where 2e-2 absolute is loose (outputs of order 0.05 on paper-shaped
+# inputs). The kernel's bf16 roundings: each softmax numerator is rounded to
+# bf16 before the PV product (relative error <= 2^-8; as the weights sum to
+# one the output moves by <= 2^-8 times the largest |v| carrying weight), and
+# the output is rounded to bf16 (<= 2^-8 |out|). When one key dominates, its
+# |v| is about |out|, so the worst case is about 2 * 2^-8 |out|; otherwise the
+# numerator errors average out over many keys. Hence
+#   max |err|  <= 2^-6 max|ref|   (twice that worst case)
+#   mean |err| <= 2^-7 mean|ref|  (round-to-nearest errors average ~2^-10 |x|)
+ATTN_MAX_REL_BF16 = 2.0 ** -6
+ATTN_MEAN_REL_BF16 = 2.0 ** -7
 LSE_RTOL = 2e-5
 CONF_RTOL = 2e-5
+
+# Figures the parity tests report besides asserting them: attention error
+# statistics per case and the number of update positions left out of the
+# exact comparison by the decision-margin protocol. conftest prints them in
+# pytest's terminal summary and writes them as JSON to $DLM_TEST_REPORT if set.
+REPORT = {"attention_errors": [], "margin_limited": []}
+
+
+def report(kind: str, **fields):
+    REPORT[kind].append(fields)
 
 
 def dev():
@@ -64,6 +81,8 @@ def check_update_margin(gpu, ref, amb, where=""):
     for b in range(g_tok.shape[0]):
         if not amb[b].any():
             assert g_ne[b] == ref[2][b], f"{where}: n_edits of sequence {b}"
+    report("margin_limited", where=where, positions=int(amb.sum()), checked=int(amb.size),
+           differing=int(diff.sum()))
     return int(amb.sum())
 
 
@@ -79,9 +98,11 @@ def check_vocab(am_gpu, conf_gpu, lse_gpu, am_ref, conf_ref, lse_ref, where=""):
 
 
 def ambiguous_positions(w: Workload, step: int, conf_ref: np.ndarray, state, argmax_ref, prompt, seqlen):
-    """Positions where a decision of the update is within the conf tolerance of
-    its boundary: |conf - tau| within CONF_RTOL, or conf within CONF_RTOL of the
-    k-th smallest response conf. Returns a bool [B, L] array."""
+    """Positions where a decision of the update could flip within the conf
+    tolerance: an edit candidate with |conf - tau| within 2 CONF_RTOL conf, or,
+    when the k-th and (k+1)-th smallest response confs are that close, every
+    position whose conf lies between them (widened by the tolerance), since
+    the remask set could then differ. Returns a bool [B, L] array."""
     return ambiguous_for(w.edit_threshold[step], w.remask_k, w.remask_frac, conf_ref, state, argmax_ref, prompt,
                          seqlen)
 
@@ -100,6 +121,9 @@ def ambiguous_for(edit_threshold, remask_k, remask_frac, conf_ref, state, argmax
         amb[b, p:n] |= edit_cand & (np.abs(c - float(tau)) <= tol)
         k = remask_count(remask_k, remask_frac, n - p)
         if 0 < k < n - p:
-            kth = np.sort(c)[k - 1]
-            amb[b, p:n] |= np.abs(c - kth) <= CONF_RTOL * max(kth, 1e-30) * 2
+            srt = np.sort(c)
+            lo, hi = srt[k - 1], srt[k]          # the last remasked and the first kept conf
+            t_lo, t_hi = 2 * CONF_RTOL * max(lo, 1e-30), 2 * CONF_RTOL * max(hi, 1e-30)
+            if hi - lo <= t_lo + t_hi:
+                amb[b, p:n] |= (c >= lo - t_lo) & (c <= hi + t_hi)
     return amb
