@@ -311,7 +311,8 @@ size_t dlm_refine_step_workspace_bytes(int64_t batch);
  *
  * - The first call on a device sets up that device: it takes the array's
  *   device address with cudaGetSymbolAddress, with that device current.
- *   Make that first call before any stream capture on the device.
+ *   Make that first call before any stream capture on the device;
+ *   dlm_loop_begin does this set-up itself, so a recorded pass may use it.
  * - Each call clears the counters it uses (an asynchronous memset on the
  *   call's stream) and then launches the fused kernel.
  * - All calls on one device share the array: calls that overlap on the GPU
@@ -346,7 +347,9 @@ int dlm_refine_step_static(const dlm_tensor* logits, const dlm_tensor* tokens, c
  *
  * dlm_loop_end builds a CUDA graph: steps = 0, then WHILE { pass; steps += 1;
  * continue iff steps < max_steps and n_edits[b] > 0 for some b < B and the
- * device error word is clear }. n_edits is the [B] int32 edit count written
+ * device error word holds no bit other than DLM_DEVERR_LENGTH }: a clamped
+ * length has a defined result, every other bit leaves the pass's outputs
+ * undefined and ends the loop. n_edits is the [B] int32 edit count written
  * by the recorded pass. The test runs on the GPU after each pass, so there is
  * no host round trip between passes. Validation failures and capture errors
  * end the capture and return an error; dlm_loop_cancel ends an unfinished
@@ -372,6 +375,20 @@ const char* dlm_status_string(int status);
 const char* dlm_last_error(void);
 /* MAJOR * 10000 + MINOR * 100 + PATCH. */
 int dlm_version(void);
+
+/*
+ * Self-test of the bounded waits; a diagnostic of this library, with no
+ * counterpart in the paper. Every pipelined kernel waits for its producers
+ * with a wait that gives up after a wall-clock budget, records
+ * DLM_DEVERR_TIMEOUT in the device error word and ends the kernel, so that a
+ * stalled pipeline cannot hang the GPU. This call launches, on the calling
+ * thread's stream, a one-thread kernel that waits through that same code, for
+ * budget_ns nanoseconds (1e3 .. 1e9), on a barrier on which nothing ever
+ * arrives. Once it has run, dlm_get_device_error reports DLM_DEVERR_TIMEOUT
+ * (a recorded refine loop whose pass makes this call stops after that pass).
+ * Returns DLM_ERR_ARG, with nothing launched, for a budget outside the range.
+ */
+int dlm_selftest_wait_timeout(int64_t budget_ns);
 
 /*
  * Reads the device error word of the current device into *bits (DLM_DEVERR_*),

@@ -1,0 +1,28 @@
+/*
+ * Test hooks exported only by DLM_CHECK_BOUNDS builds of libdlmrefine
+ * (python -m paper_2608_02625_gb300.build --check-bounds --out DIR); the
+ * default build does not have them. None of them is part of the method.
+ */
+#ifndef DLMREFINE_CHECKED_H_
+#define DLMREFINE_CHECKED_H_
+
+#include "dlmrefine.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/*
+ * Fills every byte of dlm_refine_step_static's static scratch array on the
+ * current device with `byte_value` (0..255), asynchronously on the calling
+ * thread's stream. A test sets it to a nonzero pattern to check that each
+ * static call clears the counters it uses before it counts. Returns
+ * DLM_ERR_ARG for a value outside 0..255.
+ */
+int dlm_checked_fill_static_scratch(int32_t byte_value);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DLMREFINE_CHECKED_H_ */

@@ -71,6 +71,8 @@ def _load():
     lib.dlm_loop_destroy.argtypes = [ctypes.c_void_p]
     for f in ("dlm_loop_begin", "dlm_loop_end", "dlm_loop_cancel", "dlm_loop_launch", "dlm_loop_destroy"):
         getattr(lib, f).restype = ctypes.c_int
+    lib.dlm_selftest_wait_timeout.argtypes = [ctypes.c_int64]
+    lib.dlm_selftest_wait_timeout.restype = ctypes.c_int
     lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
     lib.dlm_get_stream.restype = ctypes.c_void_p
     lib.dlm_status_string.restype = ctypes.c_char_p
@@ -315,6 +317,15 @@ def dlm_loop_end(n_edits: torch.Tensor, max_steps: int, steps_out: torch.Tensor)
 def dlm_loop_cancel():
     """Ends an unfinished recording on this thread, keeping nothing."""
     _check(lib.dlm_loop_cancel())
+
+
+def dlm_selftest_wait_timeout(budget_ns: int, device: int | None = None):
+    """Runs a kernel whose bounded wait on a barrier nothing arrives on gives
+    up after budget_ns; afterwards device_error() holds DLM_DEVERR_TIMEOUT."""
+    dev = torch.cuda.current_device() if device is None else device
+    torch.cuda.set_device(dev)
+    _check(lib.dlm_set_stream(ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)))
+    _check(lib.dlm_selftest_wait_timeout(int(budget_ns)))
 
 
 def device_error(clear: bool = True) -> int:

@@ -30,7 +30,8 @@ BUILD = os.path.join(PKG, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 LIBS = {
-    "libdlmrefine.so": ["dlm_api.cu", "attn_tc.cu", "attn_f32.cu", "vocab.cu", "update.cu", "loop.cu", "lmhead.cu"],
+    "libdlmrefine.so": ["dlm_api.cu", "attn_tc.cu", "attn_f32.cu", "vocab.cu", "update.cu", "loop.cu", "lmhead.cu",
+                        "selftest.cu"],
     "libdlmsynth.so": ["synth.cu"],
 }
 HEADERS = ["dlm_common.cuh", "dlm_internal.h", "update_impl.cuh"]

@@ -623,6 +623,10 @@ namespace {
 std::mutex g_scratch_mu;
 int32_t* g_scratch_addr[kMaxDevices] = {};
 
+}  // namespace
+
+namespace dlm {
+
 // Device address of g_dlm_step_scratch on the current device (set up on first use).
 int static_step_scratch(int32_t** out) {
   using dlm::fail;
@@ -642,7 +646,7 @@ int static_step_scratch(int32_t** out) {
   return DLM_OK;
 }
 
-}  // namespace
+}  // namespace dlm
 
 extern "C" {
 
@@ -661,10 +665,25 @@ int dlm_refine_step_static(const dlm_tensor* logits, const dlm_tensor* tokens, c
                 ua.B, DLM_STATIC_STEP_MAX_BATCH);
   if ((st = require_error_word())) return st;
   int32_t* counters = nullptr;
-  if ((st = static_step_scratch(&counters))) return st;
+  if ((st = dlm::static_step_scratch(&counters))) return st;
   cudaError_t e = cudaMemsetAsync(counters, 0, static_cast<size_t>(ua.B) * sizeof(int32_t), t_stream);
   if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "clearing the static step scratch: %s", cudaGetErrorString(e));
   return dlm::launch_vocab_step(va, ua, counters, t_stream);
 }
 
 }  // extern "C"
+
+#ifdef DLM_CHECK_BOUNDS
+#include "dlmrefine_checked.h"
+
+extern "C" int dlm_checked_fill_static_scratch(int32_t byte_value) {
+  using dlm::fail;
+  t_last_error[0] = '\0';
+  if (byte_value < 0 || byte_value > 255) return fail(DLM_ERR_ARG, "byte_value %d outside 0..255", byte_value);
+  int32_t* scratch = nullptr;
+  if (const int st = dlm::static_step_scratch(&scratch)) return st;
+  const cudaError_t e = cudaMemsetAsync(scratch, byte_value, sizeof(g_dlm_step_scratch), t_stream);
+  if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "filling the static step scratch: %s", cudaGetErrorString(e));
+  return DLM_OK;
+}
+#endif  // DLM_CHECK_BOUNDS

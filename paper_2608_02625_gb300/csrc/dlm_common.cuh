@@ -62,8 +62,6 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wall-clock budget of one bounded wait. Long enough for any legitimate wait
-// inside one launch, short enough that a broken pipeline ends quickly.
 // Keys a query row may attend to under the attention masks of dlmrefine.h:
 // [0, hi1) and [lo2, hi2) (n_b = n, p_b = p clamped to [0, n]).
 struct KeyRanges {
@@ -89,26 +87,34 @@ __host__ __device__ __forceinline__ KeyRanges key_ranges(int mode, int block, in
   return r;
 }
 
+// Wall-clock budget of one bounded wait. Long enough for any legitimate wait
+// inside one launch, short enough that a broken pipeline ends quickly.
 constexpr uint64_t kWaitBudgetNs = 2000000000ull;  // 2 s
 
 // Waits for the phase with parity `parity` of `bar` to complete. Gives up
 // (returns false) when *abort is set by another thread of the block or when
-// the budget runs out; in the latter case sets *abort and the error word.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          int* err) {
+// `budget_ns` of wall-clock time has passed; in the latter case sets *abort
+// and DLM_DEVERR_TIMEOUT in the error word.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort, int* err,
+                                              uint64_t budget_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0u) {
       if (*abort) return false;
-      if (global_timer_ns() - t0 > kWaitBudgetNs) {
+      if (global_timer_ns() - t0 > budget_ns) {
         *abort = 1;
         set_device_error(err, DLM_DEVERR_TIMEOUT);
         return false;
       }
     }
   }
+}
+
+// The bounded wait of every kernel: mbar_wait_for with the kWaitBudgetNs budget.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
+  return mbar_wait_for(bar, parity, abort, err, kWaitBudgetNs);
 }
 
 // A bounded wait that ignores the abort flag: used during teardown to let
@@ -352,6 +358,18 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
       "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
       : "=f"(d.x), "=f"(d.y)
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+// acc + (the two bf16 values of a packed pair, lo in bits 0-15) as fp32, one
+// mixed-precision add per lane (sm_100 family): the bf16 operands convert
+// exactly, each sum is rounded once.
+__device__ __forceinline__ float2 add_bf16x2_f32(float2 acc, uint32_t pk) {
+  float2 d;
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %4;\n\t"
+      "add.rn.f32.bf16 %0, lo, %2;\n\tadd.rn.f32.bf16 %1, hi, %3;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(acc.x), "f"(acc.y), "r"(pk));
   return d;
 }
 

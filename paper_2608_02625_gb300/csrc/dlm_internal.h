@@ -51,13 +51,6 @@ struct VocabArgs {
 
 int launch_vocab_confidence(const VocabArgs& a, cudaStream_t stream);
 
-// The same reduction with a caller workspace of vocab_workspace_bytes(N)
-// bytes (zero on entry, left zero): with few rows, the logits are split
-// evenly over all CTAs and each row's partials merged through the workspace.
-constexpr int kVocabFlatMaxCtas = 4096;
-constexpr int kVocabFlatMaxRowsPerCta = 8;
-size_t vocab_workspace_bytes(int64_t N);
-int launch_vocab_confidence_ws(const VocabArgs& a, void* workspace, cudaStream_t stream);
 
 struct UpdateArgs {
   const int32_t* tokens;

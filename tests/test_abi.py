@@ -312,3 +312,27 @@ def test_masked_attention_rejects():
     assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(pl), 1, 0, r(o)) == -6          # block < 1
     assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(T(I32, [3], 6 * MB)), 1, 64, r(o)) == -3
     assert lib.dlm_attn_masked(r(q), r(k), r(v), r(sl), r(T(F32, [2], 6 * MB)), 2, 64, r(o)) == -2
+
+
+def test_selftest_rejects_budget_outside_range():
+    so = ctypes.CDLL(os.path.join(PKG, "libdlmrefine.so"))
+    so.dlm_selftest_wait_timeout.argtypes = [ctypes.c_int64]
+    for budget in (0, 999, 1000000001, -5):
+        assert so.dlm_selftest_wait_timeout(budget) == -6   # DLM_ERR_ARG, nothing launched
+
+
+def test_checked_build_exports_its_test_hooks(tmp_path):
+    """A DLM_CHECK_BOUNDS build exports what dlmrefine.h and dlmrefine_checked.h
+    declare; the default build has none of the checked-only hooks."""
+    from paper_2608_02625_gb300 import build
+    build.build(check_bounds=True, out_dir=str(tmp_path))
+    checked = ctypes.CDLL(str(tmp_path / "libdlmrefine.so"))
+    default = ctypes.CDLL(os.path.join(PKG, "libdlmrefine.so"))
+    hooks = declared_functions("dlmrefine_checked.h")
+    assert hooks == ["dlm_checked_fill_static_scratch"]
+    for n in declared_functions("dlmrefine.h") + hooks:
+        assert hasattr(checked, n), f"checked build does not export {n}"
+    for n in hooks:
+        assert not hasattr(default, n), f"default build exports the test hook {n}"
+    checked.dlm_checked_fill_static_scratch.argtypes = [ctypes.c_int32]
+    assert checked.dlm_checked_fill_static_scratch(256) == -6

@@ -78,3 +78,51 @@ def test_checked_build_reports_contract_violations(tmp_path):
     torch.cuda.synchronize()
     assert err_bits(checked) & DLM_DEVERR_INPUT
     assert float(prob[5]) == 0.0
+
+
+@pytest.mark.gpu
+def test_static_step_clears_poisoned_scratch(tmp_path):
+    """dlm_refine_step_static clears the counters it uses before it counts: with
+    its static scratch filled with a nonzero pattern, a call still matches the
+    workspace call (same library) bit for bit, twice in a row."""
+    import numpy as np
+    import torch
+    from paper_2608_02625_gb300 import binding as Bn
+    from paper_2608_02625_gb300 import build
+    build.build(check_bounds=True, out_dir=str(tmp_path))
+    checked = ctypes.CDLL(str(tmp_path / "libdlmrefine.so"))
+    d = torch.device("cuda", 0)
+    torch.cuda.set_device(d)
+    stream = torch.cuda.current_stream(d)
+    assert checked.dlm_set_stream(ctypes.c_void_p(stream.cuda_stream)) == 0
+    B, L, V = 6, 96, 3000
+    g = torch.Generator().manual_seed(17)
+    logits = (torch.randn(B * L, V, generator=g) * 3).to(torch.bfloat16).to(d)
+    tok = torch.randint(0, V, (B, L), generator=g, dtype=torch.int32).to(d)
+    msk = (torch.rand(B, L, generator=g) < 0.25).to(torch.uint8).to(d)
+    prompt = torch.randint(0, 40, (B,), generator=g, dtype=torch.int32).to(d)
+    seqlen = torch.full((B,), L, dtype=torch.int32, device=d)
+    params = Bn.RefineParams(0.8, 9, 0.0, V, prompt, seqlen).to_c()
+
+    def outs():
+        return [torch.empty((B, L), dtype=t, device=d) for t in (torch.int32, torch.float32, torch.float32,
+                                                                 torch.int32, torch.uint8)] + \
+               [torch.empty(B, dtype=torch.int32, device=d)]
+
+    def descs(ts):
+        return [ctypes.byref(Bn.describe(t)) for t in ts]
+
+    ref = outs()
+    ws = torch.zeros(B, dtype=torch.int32, device=d)
+    st = checked.dlm_refine_step(*descs((logits, tok, msk)), ctypes.byref(params), *descs(ref),
+                                 ctypes.c_void_p(ws.data_ptr()), ctypes.c_size_t(4 * B))
+    assert st == 0
+    for call in range(2):
+        assert checked.dlm_checked_fill_static_scratch(0x55) == 0
+        got = outs()
+        assert checked.dlm_refine_step_static(*descs((logits, tok, msk)), ctypes.byref(params), *descs(got)) == 0
+        torch.cuda.synchronize()
+        for name, x, y in zip(("argmax", "conf", "lse", "tokens", "mask", "n_edits"), got, ref):
+            assert torch.equal(x, y), f"call {call + 1}: {name} differs from the workspace call"
+    bits = ctypes.c_int32(0)
+    assert checked.dlm_get_device_error(ctypes.byref(bits), 1) == 0 and bits.value == 0
