@@ -544,6 +544,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // Numerators 2^(s * scale - m), two columns at a time; P goes to tensor
         // memory (over the first 32 columns of this S buffer) 16 columns at a time.
+        // The row sum l adds the numerators as rounded to bf16, the values the
+        // PV product uses, so the output is an exactly normalised average of v
+        // (a key that takes all the weight yields its v unchanged).
         const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
         // A row whose keys so far were all masked keeps m_used = -inf: its
         // numerators are exp2(-inf) = 0 (subtracting 0 avoids -inf - -inf).
@@ -558,8 +561,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int col = 32 * qq + 2 * c;
             const float2 x = ffma2(make_float2(sv[col], sv[col + 1]), sc2, nm2);
             const float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
-            if (c & 1) acc1 = fadd2(acc1, e); else acc0 = fadd2(acc0, e);
             pk[c] = pack_bf16x2(e.x, e.y);
+            if (c & 1) acc1 = add_bf16x2_f32(acc1, pk[c]); else acc0 = add_bf16x2_f32(acc0, pk[c]);
           }
           tmem_st16(s_addr + 16 * qq, pk);
         }

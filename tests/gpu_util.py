@@ -21,15 +21,18 @@ ATTN_TOL_F32 = 1e-5
 # Bounds scaled to the output, which a small systematic error would break
 # even where 2e-2 absolute is loose (outputs of order 0.05 on paper-shaped
 # inputs). The kernel's bf16 roundings: each softmax numerator is rounded to
-# bf16 before the PV product (relative error <= 2^-8; as the weights sum to
-# one the output moves by <= 2^-8 times the largest |v| carrying weight), and
-# the output is rounded to bf16 (<= 2^-8 |out|). When one key dominates, its
-# |v| is about |out|, so the worst case is about 2 * 2^-8 |out|; otherwise the
-# numerator errors average out over many keys. Hence
-#   max |err|  <= 2^-6 max|ref|   (twice that worst case)
-#   mean |err| <= 2^-7 mean|ref|  (round-to-nearest errors average ~2^-10 |x|)
-ATTN_MAX_REL_BF16 = 2.0 ** -6
-ATTN_MEAN_REL_BF16 = 2.0 ** -7
+# bf16 (round to nearest even, relative error <= 2^-8) before the PV product
+# and the row sum adds the same rounded values, so the output is an exactly
+# normalised average of v with perturbed weights; the output is then rounded
+# to bf16 (<= 2^-8 |out|). The worst case is about 2 * 2^-8 |out|, and the
+# round-to-nearest errors average out. Hence, against the fp64 oracle:
+#   max |err|                  <= 2^-7  max|ref|   (measured <= 5.6e-3)
+#   mean |err|                 <= 2^-8  mean|ref|  (measured <= 2.3e-3)
+#   |mean (err * sign(ref))|   <= 2^-10 mean|ref|  (measured <= 5e-4; rounding
+#                                                   towards zero would give ~2^-9)
+ATTN_MAX_REL_BF16 = 2.0 ** -7
+ATTN_MEAN_REL_BF16 = 2.0 ** -8
+ATTN_BIAS_REL_BF16 = 2.0 ** -10
 LSE_RTOL = 2e-5
 CONF_RTOL = 2e-5
 
@@ -37,7 +40,7 @@ CONF_RTOL = 2e-5
 # statistics per case and the number of update positions left out of the
 # exact comparison by the decision-margin protocol. conftest prints them in
 # pytest's terminal summary and writes them as JSON to $DLM_TEST_REPORT if set.
-REPORT = {"attention_errors": [], "margin_limited": []}
+REPORT = {"attention_errors": [], "margin_limited": [], "notes": []}
 
 
 def report(kind: str, **fields):

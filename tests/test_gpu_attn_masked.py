@@ -1,6 +1,6 @@
 """Block-causal and block-local attention (dlm_attn_masked) on the GPU against
 the oracle's mask variants, with the tolerances of the unmasked attention
-tests: bf16 max abs error 2e-2 (+1e-2 |ref| on peaked inputs), fp32 1e-5;
+tests: bf16 max abs error 2e-2 and the output-scaled bounds, fp32 1e-5;
 rows i >= n_b exactly zero. The full mode through the same entry point must
 equal dlm_bidir_attn bit for bit."""
 import math
@@ -10,7 +10,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_util import ATTN_RTOL_PEAKED, ATTN_TOL_BF16, ATTN_TOL_F32, dev, host_qkv_seq
+from gpu_util import ATTN_TOL_BF16, ATTN_TOL_F32, dev, host_qkv_seq
 from paper_2608_02625_gb300 import workloads
 from test_gpu_attn import compare, rand_qkv
 
@@ -39,7 +39,7 @@ def run(B, L, Hq, Hkv, D, sl, pl, mode, block, sigma, dtype, seed):
     where = f"mode {mode} block {block} B{B} L{L} {Hq}/{Hkv} D{D} sl {sl} pl {pl}"
     if dtype == "f32":
         return compare(out, ref, sl, ATTN_TOL_F32, where=where)
-    return compare(out, ref, sl, ATTN_TOL_BF16, ATTN_RTOL_PEAKED if sigma >= 0.5 else 0.0, where=where)
+    return compare(out, ref, sl, ATTN_TOL_BF16, where=where + f" sigma {sigma:.3g}")
 
 
 @pytest.mark.parametrize("mode", [CAUSAL, LOCAL])
