@@ -10,7 +10,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_util import ambiguous_positions, check_vocab, dev, host_logit_rows
+from gpu_util import ambiguous_positions, check_vocab, dev, host_logit_rows, report
 from paper_2608_02625_gb300 import workloads
 
 pytestmark = pytest.mark.gpu
@@ -45,6 +45,8 @@ def compare_update(w, step, seqs, state, ref_vocab, gpu_upd, where):
                                prompt_lens=p, seq_lens=n)
     g_tok, g_msk, g_ne = gpu_upd
     amb = ambiguous_positions(w, step, cf_ref, state, am_ref, p, n)
+    report("margin_limited", where=where, positions=int(amb.sum()), checked=int(amb.size),
+           differing=int(((g_tok != ref[0]) | (g_msk != ref[1])).sum()))
     diff = (g_tok != ref[0]) | (g_msk != ref[1])
     assert not np.any(diff & ~amb), f"{where}: update differs at unambiguous positions {np.argwhere(diff & ~amb)[:8]}"
     for i in range(len(seqs)):
@@ -121,3 +123,46 @@ def test_four_step_chain():
             o_tok, o_msk = ref[0], ref[1]
             diverged = n_diff > 0   # a tolerated flip at an ambiguous position: chains part ways
         g_tok, g_msk = nt, nm
+
+
+def test_c2_literal_peak_reading():
+    """The single-sequence workload under the literal reading of its "+8
+    peaked token": the peaked token's own N(0, 3) draw plus 8 (the workloads
+    use 8 above the typical row maximum instead). The same rows are peaked and
+    the same tokens chosen; the +8 is added in fp32 and rounded to bf16 on both
+    sides. Vocabulary outputs against the oracle on every row, then the update
+    under the decision-margin protocol. Reported: how many peaked tokens end
+    up as the argmax and how many edits fire (with a +8 on one draw of 151552,
+    the token rarely beats the row maximum, and its confidence stays far below
+    the edit threshold)."""
+    from gpu_util import report
+    from paper_2608_02625_gb300 import synth, synth_gpu
+    w = workloads.scaled(workloads.get("c2_single_512"), peak_frac=(0.0,))     # plain N(0, 3) draws
+    base = workloads.get("c2_single_512")
+    d = dev()
+    rows = np.arange(w.N)
+    is_peak, ptok, _ = base.logit_spec(0).peak_plan(rows)
+    pr, pt = rows[is_peak], ptok[is_peak].astype(np.int64)
+    logits = synth_gpu.logits(w, 0, d)
+    r_t, t_t = torch.from_numpy(pr).to(d), torch.from_numpy(pt).to(d)
+    logits[r_t, t_t] = (logits[r_t, t_t].float() + 8.0).to(torch.bfloat16)
+    host = host_logit_rows(w, 0, rows)
+    host[pr, pt] = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits((host[pr, pt] + np.float32(8.0)).astype(np.float32)))
+    assert np.array_equal(logits.float().cpu().numpy(), host)
+    tok, msk = w.initial_state()
+    q, k, v = synth_gpu.qkv(w, 0, d)
+    prompt = torch.from_numpy(w.prompt_lens()).to(d)
+    seqlen = torch.from_numpy(w.seq_lens()).to(d)
+    _, am, cf, ls, nt, nm, ne = gpu_step(w, 0, q, k, v, logits, torch.from_numpy(tok).to(d),
+                                         torch.from_numpy(msk).to(d), prompt, seqlen)
+    ref_vocab = oracle.vocab_confidence(host)
+    check_vocab(am.cpu().numpy(), cf.cpu().numpy(), ls.cpu().numpy(), *ref_vocab, where="c2 literal +8")
+    ref_v = tuple(a.reshape(1, w.L) for a in ref_vocab)
+    g = (nt.cpu().numpy(), nm.cpu().numpy(), ne.cpu().numpy())
+    ref, n_amb, _ = compare_update(w, 0, [0], (tok, msk), ref_v, g, "c2 literal +8")
+    report("margin_limited", where="c2_single_512 literal +8 reading", positions=n_amb, checked=w.L,
+           differing=int(((g[0] != ref[0]) | (g[1] != ref[1])).sum()))
+    wins = int(np.sum(ref_vocab[0][pr] == pt))
+    report("notes", text=f"c2 literal +8 reading: {wins} of {len(pr)} peaked tokens are the argmax, "
+                         f"{int(ref[2][0])} edits, largest confidence {float(ref_vocab[1].max()):.3g}")
+    assert int(ne[0]) == int(ref[2][0])

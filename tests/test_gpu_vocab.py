@@ -131,3 +131,40 @@ def test_split_rows_several_per_cluster(dtype, N, V):
     ref = oracle.vocab_confidence(t.float().cpu().numpy())
     check_vocab(am, cf, ls, *ref, where=f"{dtype} {N}x{V}")
     assert all(am[r] == chunk - 1 for r in range(0, N, 7))
+
+
+def test_c4_zipf_full_size_planted_ties():
+    """The long-draft workload at full size (16384 rows of the Zipf(1.1) prior
+    plus N(0, 1)), with equal maxima planted in sampled rows at positions that
+    fall to different threads, warps and staging slots of the row kernel, and
+    to different CTAs' chunks of the split-row clusters (a 256-row slice); the
+    lowest index must win everywhere."""
+    from paper_2608_02625_gb300 import synth_gpu
+    w = workloads.get("c4_long_2048")
+    x = synth_gpu.logits(w, 0, dev())
+    V = w.V
+    rng = np.random.default_rng(44)
+    rows = np.unique(np.concatenate([[0, 1, 255, w.N - 1], rng.integers(0, w.N, 24)]))
+    pos = np.array([V // 8 - 1, 3 * (V // 8) + 5, V // 2 + 2048 * 8 + 3, V - 1])   # first planted index wins
+    peak = float(x[torch.from_numpy(rows).to(dev())].float().max().item()) + 16.0   # exact in bf16 (an integer)
+    peak = float(torch.tensor(peak).to(torch.bfloat16).float())
+    for r in rows:
+        x[int(r), torch.from_numpy(pos).to(dev())] = peak
+    am, cf, ls = gpu_vocab(x)
+    ref = oracle.vocab_confidence(host_rows_planted(w, rows, pos, peak))
+    check_vocab(am[rows], cf[rows], ls[rows], *ref, where="c4 planted ties")
+    assert np.all(am[rows] == pos[0])
+    sl = rows[rows < 256]
+    sub = x[:256]
+    ref_s = oracle.vocab_confidence(host_rows_planted(w, sl, pos, peak))
+    outs = gpu_vocab(sub)
+    check_vocab(outs[0][sl], outs[1][sl], outs[2][sl], *ref_s, where="c4 planted ties, 256 rows, clusters")
+    assert np.all(outs[0][sl] == pos[0])
+    del x
+    torch.cuda.empty_cache()
+
+
+def host_rows_planted(w, rows, pos, peak):
+    x = host_logit_rows(w, 0, rows)
+    x[:, pos] = np.float32(peak)
+    return x
