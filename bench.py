@@ -55,33 +55,93 @@ def load_peaks():
 # ---------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """Samples nvidia-smi SM clocks and throttle reasons during the timed region."""
+    """Samples the SM clock and the throttle reasons during the timed region.
+
+    Read-only queries only. Through NVML (the driver's libnvidia-ml, via
+    ctypes) every 2 ms when it loads, so that even a region of ~20 ms carries
+    several samples; otherwise nvidia-smi's own loop every 5 ms."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    # NVML clock event reason bits
+    REASON_BITS = {"sw_power_cap": 0x4, "hw_slowdown": 0x8, "sw_thermal_slowdown": 0x20,
+                   "hw_thermal_slowdown": 0x40}
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, pci_bus_id: str | None = None):
         self.gpu = gpu_index
+        self.pci = pci_bus_id
         self.proc = None
-        self.lines = []
+        self.samples = []     # (host time, sm_mhz, sm_max_mhz, set of active reason names)
+        self.source = None
+        self._stop = threading.Event()
+
+    def _nvml(self):
+        import ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            return None
+        h = ctypes.c_void_p()
+        if not (self.pci and lib.nvmlDeviceGetHandleByPciBusId_v2(self.pci.encode(), ctypes.byref(h)) == 0):
+            if lib.nvmlDeviceGetHandleByIndex_v2(self.gpu, ctypes.byref(h)) != 0:
+                return None
+        reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        mhz, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+
+        def poll():
+            if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz)) != 0:   # NVML_CLOCK_SM
+                return None
+            lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx))
+            reasons_fn(h, ctypes.byref(rs))
+            return (float(mhz.value), float(mx.value),
+                    {n for n, bit in self.REASON_BITS.items() if rs.value & bit})
+        return poll if poll() is not None else None
 
     def __enter__(self):
+        poll = None
+        try:
+            poll = self._nvml()
+        except Exception:
+            poll = None
+        if poll is not None:
+            self.source = "nvml every 2 ms"
+
+            def run():
+                while not self._stop.is_set():
+                    r = poll()
+                    if r is not None:
+                        self.samples.append((time.time(),) + r)
+                    time.sleep(0.002)
+            self.thread = threading.Thread(target=run, daemon=True)
+            self.thread.start()
+            return self
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                          "--format=csv,noheader,nounits", "-lms", "5"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.source = "nvidia-smi -lms 5"
+            self.thread = threading.Thread(target=self._read_smi, daemon=True)
             self.thread.start()
         except Exception:
             self.proc = None
         return self
 
-    def _read(self):
+    def _read_smi(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in self.proc.stdout:
-            self.lines.append((time.time(), line.strip()))
+            parts = [x.strip() for x in line.strip().split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm, mx = float(parts[1]), float(parts[2])
+            except ValueError:
+                continue
+            active = {nm for nm, val in zip(names, parts[5:9]) if val.lower().startswith("active")}
+            self.samples.append((time.time(), sm, mx, active))
 
     def __exit__(self, *exc):
+        self._stop.set()
         if self.proc:
             self.proc.terminate()
             try:
@@ -92,29 +152,19 @@ class ClockSampler:
     def summary(self, t0=None, t1=None):
         """Median SM clock and active throttle reasons of the samples taken in
         [t0, t1] (host time); all samples if the window caught none."""
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        lines = [ln for ts, ln in self.lines if t0 is None or t0 <= ts <= t1]
+        win = [x for x in self.samples if t0 is None or t0 <= x[0] <= t1]
         window = "timed region"
-        if not lines:
-            lines = [ln for _, ln in self.lines]
+        if not win:
+            win = list(self.samples)
             window = "whole run (no sample inside the timed region)"
-        for ln in lines:
-            parts = [x.strip() for x in ln.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                mx.append(float(parts[2]))
-            except ValueError:
-                continue
-            for nm, val in zip(names, parts[5:9]):
-                if val.lower().startswith("active"):
-                    reasons.add(nm)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm), "window": window}
+        if not win:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "source": self.source}
+        reasons = set()
+        for x in win:
+            reasons |= x[3]
+        return {"sm_mhz": statistics.median(x[1] for x in win), "sm_max_mhz": max(x[2] for x in win),
+                "sm_mhz_min": min(x[1] for x in win), "reasons": sorted(reasons), "samples": len(win),
+                "window": window, "source": self.source}
 
 
 # ---------------------------------------------------------------- traffic record
@@ -143,58 +193,59 @@ def recorded_traffic(kernel_file: str, kernel: str, workload: str):
 
 # ---------------------------------------------------------------- CPU oracle timing
 
-def _oracle_worker(conn, name, b, vocab_rows):
-    """A host core timing the oracle on sequence b of the workload: fp64
-    attention over every head, the vocabulary reduction of `vocab_rows` of its
-    rows (spread over the sequence), and the update of the whole sequence.
-    Inputs are generated once, before any timing."""
+def _oracle_worker(conn, name, seqs):
+    """A host core running the oracle on whole sequences `seqs` of the
+    workload: fp64 attention over every head, the vocabulary reduction of
+    every row, and the update of the sequence from those predictions. Inputs
+    are generated once, before any timing."""
     import numpy as np
     import oracle
     from paper_2608_02625_gb300 import synth, workloads
     w = workloads.get(name)
+    tok, msk = w.initial_state()
+    n_all, p_all = w.seq_lens(), w.prompt_lens()
 
-    def host(which, H):
+    def host(b, which, H):
         per = w.L * H * w.D
         x = synth.qkv_host(w.seed, which, (w.B, w.L, H, w.D), w.qkv_sigma, w.dtype, b * per, per)
         x = synth.bf16_bits_to_f32(x) if w.dtype == "bf16" else x
         return x.reshape(1, w.L, H, w.D)
 
-    q, k, v = host(synth.S_Q, w.Hq), host(synth.S_K, w.Hkv), host(synth.S_V, w.Hkv)
-    tok, msk = w.initial_state()
-    rows = b * w.L + np.linspace(0, w.L - 1, vocab_rows).astype(np.int64)
-    x = w.logit_spec(0).rows_f32(rows, tok.reshape(-1)[rows], msk.reshape(-1)[rows])
-    if w.dtype == "bf16":
-        x = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(x))
-    # The update reads a full sequence of predictions; the sampled rows' values
-    # are tiled over it (the update's cost does not depend on the values).
-    reps = -(-w.L // vocab_rows)
-    n, p = w.seq_lens()[b:b + 1], w.prompt_lens()[b:b + 1]
+    inputs = []
+    for b in seqs:
+        rows = np.arange(b * w.L, (b + 1) * w.L)
+        x = w.logit_spec(0).rows_f32(rows, tok.reshape(-1)[rows], msk.reshape(-1)[rows])
+        if w.dtype == "bf16":
+            x = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(x))
+        inputs.append((b, host(b, synth.S_Q, w.Hq), host(b, synth.S_K, w.Hkv), host(b, synth.S_V, w.Hkv), x))
     conn.send("ready")
     while conn.recv() == "run":
-        t0 = time.perf_counter()
-        oracle.bidir_attn(q, k, v, n)
-        t1 = time.perf_counter()
-        am, cf, _ = oracle.vocab_confidence(x)
-        t2 = time.perf_counter()
-        oracle.refine_update(tok[b:b + 1], msk[b:b + 1], np.tile(am, reps)[None, :w.L],
-                             np.tile(cf, reps)[None, :w.L], edit_threshold=w.edit_threshold[0],
-                             remask_k=w.remask_k, remask_frac=w.remask_frac, mask_id=w.mask_id,
-                             prompt_lens=p, seq_lens=n)
-        t3 = time.perf_counter()
-        conn.send((t1 - t0, (t2 - t1) * w.L / vocab_rows, t3 - t2))
+        t = [0.0, 0.0, 0.0]
+        for b, q, k, v, x in inputs:
+            t0 = time.perf_counter()
+            oracle.bidir_attn(q, k, v, n_all[b:b + 1])
+            t1 = time.perf_counter()
+            am, cf, _ = oracle.vocab_confidence(x)
+            t2 = time.perf_counter()
+            oracle.refine_update(tok[b:b + 1], msk[b:b + 1], am[None, :], cf[None, :],
+                                 edit_threshold=w.edit_threshold[0], remask_k=w.remask_k, remask_frac=w.remask_frac,
+                                 mask_id=w.mask_id, prompt_lens=p_all[b:b + 1], seq_lens=n_all[b:b + 1])
+            t3 = time.perf_counter()
+            t = [t[0] + t1 - t0, t[1] + t2 - t1, t[2] + t3 - t2]
+        conn.send(tuple(t))
 
 
 class OracleTimer:
-    """Single-threaded processes (spawned, at most one per sequence of the
-    batch), each timing one sequence."""
-
-    VOCAB_ROWS = 64
+    """The oracle on the whole batch of a workload, spread over the host cores:
+    single-threaded processes (spawned; at most one per sequence), each owning
+    whole sequences (sequence b goes to process b mod P). One round is one
+    refine step of the whole batch, and its time is the wall time until the
+    last process is done."""
 
     def __init__(self, name: str, workers: int):
         from paper_2608_02625_gb300 import workloads
         self.w = workloads.get(name)
         self.name = name
-        # No more workers than sequences: a step has B sequences to spread.
         workers = max(1, min(workers, self.w.B))
         os.environ["OPENBLAS_NUM_THREADS"] = "1"
         os.environ["OMP_NUM_THREADS"] = "1"
@@ -202,8 +253,8 @@ class OracleTimer:
         self.conns, self.procs = [], []
         for i in range(workers):
             a, bconn = ctx.Pipe()
-            pr = ctx.Process(target=_oracle_worker, args=(bconn, name, (i * 7) % self.w.B, self.VOCAB_ROWS),
-                             daemon=True)
+            seqs = list(range(i, self.w.B, workers))
+            pr = ctx.Process(target=_oracle_worker, args=(bconn, name, seqs), daemon=True)
             pr.start()
             self.conns.append(a)
             self.procs.append(pr)
@@ -218,23 +269,21 @@ class OracleTimer:
             self.ready = True
 
     def run(self):
-        """One round: every worker times its sequence. Returns cpu_baseline."""
+        """One refine step of the whole batch on the oracle. Returns cpu_baseline."""
         self.wait_ready()
+        t0 = time.perf_counter()
         for c in self.conns:
             c.send("run")
         parts = [c.recv() for c in self.conns]
-        per_seq = [sum(x) for x in parts]
-        mean_seq = statistics.mean(per_seq)
+        wall = time.perf_counter() - t0
         w = self.w
         cores = len(self.conns)
-        return {"value": cores / (mean_seq * w.B), "unit": UNIT, "cores": cores, "kind": "oracle",
-                "sample": (f"{cores} of the {w.B} sequences of {self.name}, one per single-threaded process: "
-                           f"fp64 attention over all {w.Hq} heads, vocabulary reduction of {self.VOCAB_ROWS} of "
-                           f"its {w.L} rows scaled to {w.L}, update of the whole sequence; "
-                           f"steps/s = cores / (B x mean seconds per sequence)"),
-                "oracle_s_per_sequence": {"attn": statistics.mean(x[0] for x in parts),
-                                          "vocab": statistics.mean(x[1] for x in parts),
-                                          "update": statistics.mean(x[2] for x in parts)}}
+        return {"value": 1.0 / wall, "unit": UNIT, "cores": cores, "kind": "oracle", "ms_per_step": wall * 1e3,
+                "sample": (f"the whole batch of {self.name} ({w.B} sequences, all {w.Hq} heads, all {w.L} "
+                           f"vocabulary rows of {w.V}), one step, on {cores} single-threaded processes owning "
+                           f"whole sequences; steps/s = 1 / wall time of the step"),
+                "oracle_cpu_s_per_step": {"attn": sum(x[0] for x in parts), "vocab": sum(x[1] for x in parts),
+                                          "update": sum(x[2] for x in parts)}}
 
     def close(self):
         for c in self.conns:
@@ -247,7 +296,7 @@ class OracleTimer:
 
 
 def host_workers():
-    return max(1, min(16, (os.cpu_count() or 2) - 1))
+    return max(1, min(64, os.cpu_count() or 1))
 
 
 # ---------------------------------------------------------------- multi-GPU (replicas)
@@ -554,6 +603,203 @@ def measure_e2e(args, Bn, w, bufs, stream, mask_mode, world, d, copy_streams=4):
             "copies": f"{copy_streams} copy streams, two device input sets (copies of step s+1 overlap step s)"}
 
 
+L2_BYTES = 129 * 1024 * 1024
+
+
+def pci_bus_id(d):
+    """NVML's PCI bus id of torch device d, or None if torch does not expose it."""
+    try:
+        import torch
+        pr = torch.cuda.get_device_properties(d)
+        return f"{pr.pci_domain_id:08x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+    except Exception:
+        return None
+
+
+def timed_launches(fn_of_set, nsets: int, reps: int, stream, warm: int = 3):
+    """Mean device time (ms) per launch of fn_of_set(i % nsets), i < reps.
+
+    The launches are captured once into a CUDA graph and the graph is replayed
+    between two CUDA events: a short kernel timed eagerly would include the
+    host's time to issue it (the binding takes ~10 us per call), while the
+    graph hands the launches to the GPU back to back."""
+    import torch
+    for i in range(warm):
+        fn_of_set(i % nsets)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream(stream.device)
+    side.wait_stream(stream)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side, capture_error_mode="thread_local"):
+        for i in range(reps):
+            fn_of_set(i % nsets)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(side):   # the graph runs on the current stream
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(side)
+        g.replay()
+        e1.record(side)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def measure_workload_kernels(Bn, name: str, d, peaks, reps: int = 20):
+    """The three kernels of one refine step of workload `name`, each timed on its
+    own (CUDA events around each of `reps` launches). Inputs come from the seeded
+    generator, resident in HBM; when one set of inputs fits in L2, enough copies
+    rotate (at least three times the L2 together) that every launch reads HBM."""
+    import torch
+    from paper_2608_02625_gb300 import synth_gpu, workloads
+    w = workloads.get(name)
+    stream = torch.cuda.current_stream(d)
+    qkv_bytes = 2 * w.B * w.L * (w.Hq + 2 * w.Hkv) * w.D
+    per_set = w.logit_bytes() + qkv_bytes
+    nsets = max(1, min(4, -(-3 * L2_BYTES // per_set)))
+    tok_np, msk_np = w.initial_state()
+    tok = torch.from_numpy(tok_np).to(d)
+    msk = torch.from_numpy(msk_np).to(d)
+    q, k, v = synth_gpu.qkv(w, 0, d)
+    logits = synth_gpu.logits(w, 0, d, tok.view(-1), msk.view(-1))
+    sets = [(q, k, v, logits)] + [tuple(t.clone() for t in (q, k, v, logits)) for _ in range(nsets - 1)]
+    prompt = torch.from_numpy(w.prompt_lens()).to(d)
+    seqlen = torch.from_numpy(w.seq_lens()).to(d)
+    out = torch.empty_like(q)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, prompt, seqlen)
+    clk = ClockSampler(d.index or 0, pci_bus_id(d)).__enter__()
+    t0 = time.time()
+    t_attn = timed_launches(lambda i: Bn.dlm_bidir_attn(sets[i][0], sets[i][1], sets[i][2], seqlen, out),
+                            nsets, reps, stream)
+    t_vocab = timed_launches(lambda i: Bn.dlm_vocab_confidence(sets[i][3], am, cf, ls), nsets, reps, stream)
+    t_upd = timed_launches(lambda i: Bn.dlm_refine_update(tok, msk, am.view(w.B, w.L), cf.view(w.B, w.L), params,
+                                                          nt, nm, ne), 1, reps, stream)
+    t1 = time.time()
+    clk.__exit__(None, None, None)
+    if Bn.device_error(clear=True):
+        raise RuntimeError(f"device error word set while timing {name}")
+    flops = w.attn_flops()
+    vb = w.vocab_bytes()
+    step = t_attn + t_vocab + t_upd
+    res = {"batch": w.B, "seq_len": w.L, "q_heads": w.Hq, "kv_heads": w.Hkv, "vocab": w.V,
+           "attn": {"ms": t_attn, "tflops": flops / (t_attn * 1e-3) / 1e12,
+                    "frac_of_measured_bf16": flops / (t_attn * 1e-3) / 1e12 / peaks["bf16_tflops"]},
+           "vocab": {"ms": t_vocab, "gbs": vb / (t_vocab * 1e-3) / 1e9,
+                     "frac_of_measured_hbm": vb / (t_vocab * 1e-3) / 1e9 / peaks["hbm_gbs"]},
+           "update": {"ms": t_upd},
+           "step_ms": step, "steps_per_s": 1000.0 / step,
+           "refined_tokens_per_s": 1000.0 / step * w.refined_tokens(),
+           "note": (f"kernels timed one by one, {reps} launches each replayed from a CUDA graph after 3 warm-ups; "
+                    f"{nsets} rotating input "
+                    f"set(s) ({'L2 flushed by rotation' if nsets > 1 else 'inputs larger than L2'}); step = "
+                    f"attention + vocabulary reduction + update" + (" (step 0 of 4)" if w.steps > 1 else "")),
+           "clocks": clk.summary(t0, t1)}
+    del sets, logits, q, k, v
+    torch.cuda.empty_cache()
+    return res
+
+
+def measure_e2e_lmhead(args, Bn, w, world, d, reps: int = 20):
+    """One refine step end to end through the public API starting from the
+    refiner's last hidden states instead of materialised logits: every step
+    copies q, k, v, the hidden states [N, d] and the token state from pinned
+    host memory, runs attention, the fused vocabulary projection + reduction
+    (output weights resident, as a model's parameters are) and the update, and
+    reads the new tokens, mask and edit counts back."""
+    import torch
+    from paper_2608_02625_gb300 import synth, synth_gpu
+    stream = torch.cuda.current_stream(d)
+    dm = args.lmhead_d
+    q, k, v = synth_gpu.qkv(w, 0, d)
+    hidden = torch.empty((w.N, dm), dtype=torch.bfloat16, device=d)
+    weight = torch.empty((w.V, dm), dtype=torch.bfloat16, device=d)
+    synth_gpu.fill_normal_(hidden, synth.stream_key(w.seed + 101, synth.S_Q), 1.0)
+    synth_gpu.fill_normal_(weight, synth.stream_key(w.seed + 101, synth.S_K), 1.0 / dm ** 0.5)
+    tok_np, msk_np = w.initial_state()
+    dev_in = {"q": q, "k": k, "v": v, "hidden": hidden, "tok": torch.from_numpy(tok_np).to(d),
+              "msk": torch.from_numpy(msk_np).to(d), "prompt": torch.from_numpy(w.prompt_lens()).to(d),
+              "seqlen": torch.from_numpy(w.seq_lens()).to(d)}
+    names = list(dev_in)
+    host = {}
+    for n in names:
+        host[n] = torch.empty(dev_in[n].shape, dtype=dev_in[n].dtype, pin_memory=True)
+        host[n].copy_(dev_in[n])
+    sets = [dev_in, {n: torch.empty_like(dev_in[n]) for n in names}]
+    out = torch.empty_like(q)
+    am = torch.empty(w.N, dtype=torch.int32, device=d)
+    cf = torch.empty(w.N, dtype=torch.float32, device=d)
+    ls = torch.empty(w.N, dtype=torch.float32, device=d)
+    lws = torch.empty(Bn.dlm_lmhead_workspace_bytes(w.N), dtype=torch.uint8, device=d)
+    outs = [{"nt": torch.empty_like(dev_in["tok"]), "nm": torch.empty_like(dev_in["msk"]),
+             "ne": torch.empty(w.B, dtype=torch.int32, device=d)} for _ in range(2)]
+    h_out = [{n: torch.empty(o[n].shape, dtype=o[n].dtype, pin_memory=True) for n in o} for o in outs]
+    h2d = sum(host[n].numel() * host[n].element_size() for n in names)
+    d2h = sum(t.numel() * t.element_size() for t in h_out[0].values())
+    cstream = torch.cuda.Stream(d)
+    free = [torch.cuda.Event(), torch.cuda.Event()]
+    used = [False, False]
+
+    def copy_in(i):
+        if used[i]:
+            cstream.wait_event(free[i])
+        with torch.cuda.stream(cstream):
+            for n in names:
+                sets[i][n].copy_(host[n], non_blocking=True)
+        e = torch.cuda.Event()
+        e.record(cstream)
+        return e
+
+    def step(i):
+        st = sets[i]
+        params = Bn.RefineParams(w.edit_threshold[0], w.remask_k, w.remask_frac, w.mask_id, st["prompt"],
+                                 st["seqlen"])
+        Bn.dlm_bidir_attn(st["q"], st["k"], st["v"], st["seqlen"], out)
+        Bn.dlm_lmhead_confidence(st["hidden"], weight, am, cf, ls, lws)
+        Bn.dlm_refine_update(st["tok"], st["msk"], am.view(w.B, w.L), cf.view(w.B, w.L), params, outs[i]["nt"],
+                             outs[i]["nm"], outs[i]["ne"])
+
+    def run(nsteps):
+        pending = copy_in(0)
+        for s_ in range(nsteps):
+            i = s_ & 1
+            stream.wait_event(pending)
+            if s_ + 1 < nsteps:
+                nxt = copy_in(1 - i)
+            step(i)
+            free[i].record(stream)
+            used[i] = True
+            for n in outs[i]:
+                h_out[i][n].copy_(outs[i][n], non_blocking=True)
+            if s_ + 1 < nsteps:
+                pending = nxt
+
+    run(10)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    run(reps)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    te = max_over_ranks(e0.elapsed_time(e1) / reps, world, d)
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the hidden-state end-to-end measurement")
+    del sets, dev_in, host, weight, hidden
+    torch.cuda.empty_cache()
+    return {"value": job_steps_per_s(te, world), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": te, "steps": reps, "d_model": dm,
+            "path": "host q/k/v + hidden states -> dlm_bidir_attn -> dlm_lmhead_confidence -> dlm_refine_update "
+                    "-> host tokens/mask/edit counts (output weights resident); copies of step s+1 overlap step s"}
+
+
 def run_ours(args, rank, world):
     import numpy as np
     import torch
@@ -595,7 +841,7 @@ def run_ours(args, rank, world):
         # The workers' input generation would compete with the host-link copies
         # of the end-to-end leg: let it finish before anything is timed.
         timer.wait_ready()
-    clk = ClockSampler(d.index if d.index is not None else 0).__enter__()
+    clk = ClockSampler(d.index if d.index is not None else 0, pci_bus_id(d)).__enter__()
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -638,7 +884,13 @@ def run_ours(args, rank, world):
 
     # ---- multi-pass refinement: the recorded pass repeated by one graph launch
     # (device-side early stop) against the same passes driven from the host
+    # The other workloads first: the projection GEMM below draws enough power
+    # to leave the clocks under the power cap for a while after it.
+    by_workload = {}
+    for name in [x for x in args.workloads.split(",") if x and not args.batch]:
+        by_workload[name] = measure_workload_kernels(Bn, name, d, peaks)
     lmhead_info = measure_lmhead(args, w, Bn, peaks) if args.lmhead_d > 0 else None
+    e2e_lm = None if (args.no_e2e or args.lmhead_d <= 0) else measure_e2e_lmhead(args, Bn, w, world, d)
     loop_info = None
     if args.loop_steps > 0:
         loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
@@ -696,6 +948,8 @@ def run_ours(args, rank, world):
         "e2e": e2e,
         "loop": loop_info,
         "lmhead": lmhead_info,
+        "e2e_lmhead": e2e_lm,
+        "kernels_by_workload": by_workload,
         "paper_context": PAPER_CONTEXT,
     }
     if timer is not None:
@@ -707,26 +961,33 @@ def run_ours(args, rank, world):
 
 
 def run_reference(args, rank, world):
-    """The oracle as the reference arm: each step is one round of the host
-    cores timing their sample of the same workload, scaled to steps/s."""
+    """The oracle as the reference arm: each step is one refine step of the
+    whole batch of the workload on the host cores (see OracleTimer); the
+    step time is the wall time that passed."""
     if rank != 0:
         return None
-    timer = OracleTimer(args.config, host_workers())
-    for _ in range(args.warmup):
-        timer.run()
-    vals = [timer.run() for _ in range(args.steps)]
-    timer.close()
-    value = statistics.mean(v["value"] for v in vals)
     from paper_2608_02625_gb300 import workloads
     w = workloads.get(args.config)
+    timer = OracleTimer(args.config, host_workers())
+    timer.wait_ready()
+    for _ in range(args.warmup):
+        timer.run()
+    t0 = time.perf_counter()
+    vals = [timer.run() for _ in range(args.steps)]
+    wall = time.perf_counter() - t0
+    timer.close()
+    ms_per_step = wall * 1e3 / args.steps
+    value = 1000.0 / ms_per_step
     cb = dict(vals[-1])
     cb["value"] = value
+    cb["ms_per_step"] = ms_per_step
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value, "higher_is_better": True,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "batch": w.B, "seq_len": w.L, "q_heads": w.Hq, "kv_heads": w.Hkv,
                        "head_dim": w.D, "vocab": w.V},
             "refined_tokens_per_sec": value * w.refined_tokens(),
+            "timed_region_s": wall,
             "cpu_baseline": cb, "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                                         "d2h_bytes_per_step": 0}}
 
@@ -747,6 +1008,8 @@ def main():
     ap.add_argument("--path", default="separate", choices=["fused", "separate"],
                     help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
                          "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")
+    ap.add_argument("--workloads", default="c2_single_512,c4_long_2048,c5_heavy_4step",
+                    help="other workloads whose three kernels are also timed one by one (comma list; '' to skip)")
     ap.add_argument("--lmhead-d", type=int, default=2048,
                     help="also time the vocabulary projection fused with the reduction at this width (0: skip)")
     ap.add_argument("--attn-mask", default="full", choices=["full", "block_causal", "block_local"],

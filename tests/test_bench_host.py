@@ -82,3 +82,19 @@ def test_reference_arm_json_line():
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] == 1  # c1 has one sequence
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     assert d["config"]["workload"] == "c1_tiny_f32"
+    # A step is the whole batch and its time is time that passed.
+    assert abs(d["ms_per_step"] * d["steps"] - d["timed_region_s"] * 1e3) <= 1e-6 * d["timed_region_s"] * 1e3
+    assert "whole batch" in cb["sample"]
+
+
+def test_clock_summary_window_and_reasons():
+    """The clock record keeps the samples inside the timed region (all samples
+    when none fell inside), the median SM clock and every active reason."""
+    c = bench.ClockSampler(0)
+    c.samples = [(1.0, 1500.0, 2070.0, set()), (2.0, 2070.0, 2070.0, {"sw_power_cap"}),
+                 (2.5, 2060.0, 2070.0, set()), (3.0, 2070.0, 2070.0, {"hw_slowdown"}), (9.0, 900.0, 2070.0, set())]
+    s = c.summary(1.9, 3.1)
+    assert s["samples"] == 3 and s["sm_mhz"] == 2070.0 and s["sm_mhz_min"] == 2060.0
+    assert s["reasons"] == ["hw_slowdown", "sw_power_cap"] and s["window"] == "timed region"
+    s = c.summary(4.0, 5.0)
+    assert s["samples"] == 5 and s["window"].startswith("whole run")
