@@ -21,9 +21,12 @@
 // Warp roles (352 threads):
 //   warps 0-3  softmax + epilogue of slot 0 (thread t owns query row t = TMEM lane t)
 //   warps 4-7  softmax + epilogue of slot 1
-//   warp 8     TMA producer: Q per unit and slot; K_0, K_1, V_0, K_2, V_1, K_3, ...
-//              through a ring of eight sub-tile slots, each released as soon as
-//              the MMAs that read it have completed
+//   warp 8     TMA producer: Q per unit and slot; then the unit's key/value
+//              sub-tiles through a ring of four entries of two sub-tiles each,
+//              in the order the issuers consume them -- [K_0 | K_1], then
+//              [V_j | K_{j+2}] for each j -- so that each step of an issuer
+//              waits for one fill and releases one entry; an entry is
+//              released as soon as the MMAs that read it have completed
 //   warp 9     tensor-memory allocator; MMA issuer of slot 0 (one lane elected
 //              per instruction)
 //   warp 10    MMA issuer of slot 1
@@ -65,7 +68,7 @@ namespace {
 
 constexpr int kTile = 128;          // query rows per tile
 constexpr int kSub = 64;            // keys per sub-tile
-constexpr int kRing = 8;            // K/V ring slots (one sub-tile each)
+constexpr int kRing = 4;            // K/V ring entries (two sub-tiles each)
 constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp0 = 9;   // warps 9 and 10 issue the MMAs of slots 0 and 1
@@ -80,7 +83,7 @@ struct Smem {
   static constexpr int kKvBytes = kSub * D * 2;
   static constexpr int kStageBytes = 32 * 32 * 2;      // epilogue staging: 32 rows x 32 bf16
   alignas(1024) uint8_t q[2][kQBytes];
-  alignas(1024) uint8_t ring[kRing][kKvBytes];         // K_0, K_1, V_0, K_2, V_1, ...
+  alignas(1024) uint8_t ring[kRing][2][kKvBytes];      // [K_0 | K_1], [V_0 | K_2], [V_1 | K_3], ...
   alignas(1024) uint8_t stage[8][2][kStageBytes];       // per softmax warp, double-buffered
   uint64_t bar_q[2];          // query tile of slot i landed          (TMA -> MMA)
   uint64_t bar_qfree[2];      // last score MMA of slot i completed   (MMA -> TMA)
@@ -177,9 +180,10 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
   return U;
 }
 
-// Ring fill order of a unit with nkv sub-tiles: K_0, K_1, then for each j:
-// V_j followed by K_{j+2} (when it exists). The producer and the MMA issuer
-// walk the same order.
+// Ring entries of a unit with nkv sub-tiles: [K_0 | K_1] (K_1 when nkv > 1),
+// then for each j the entry [V_j | K_{j+2}] (K_{j+2} when it exists), which
+// holds the two tiles one step of an issuer reads: PV(j) and S(j + 2). The
+// producer and the MMA issuers walk the same order.
 
 // Warp-uniform bounded wait: true only if every lane saw the phase complete.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
@@ -253,17 +257,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tv);
       prefetch_tmap(&to);
     }
-    // Loads K_j (is_v false) or V_j into the next ring slot.
-    auto fill = [&](const Unit& U, int j, bool is_v) -> bool {
+    // Loads one ring entry: part 0 = K_ja (prologue) or V_ja, part 1 = K_jb
+    // (jb < 0: none), completing bar_full of the entry once.
+    auto load_kv = [&](uint8_t* dst, const CUtensorMap* m, uint64_t* bar, int key0, const Unit& U) {
+      for (int c = 0; c < kBoxes; ++c) tma_load_4d(dst + c * kKvBoxBytes, m, bar, 64 * c, U.g, key0, U.b);
+    };
+    auto fill = [&](const Unit& U, int ja, bool a_is_v, int jb) -> bool {
       const int r = fills % kRing;
       if (fills >= kRing && !warp_wait(&sm.bar_empty[r], ((fills / kRing) - 1) & 1, abort, p.err)) return false;
-      const int key0 = (kMasked ? U.kt(j) : j) * kSub;
-      const int valid = U.n - key0;
-      if (!is_v || valid >= kSub) {
+      const int key_a = (kMasked ? U.kt(ja) : ja) * kSub;
+      const int key_b = jb >= 0 ? (kMasked ? U.kt(jb) : jb) * kSub : 0;
+      const uint32_t b_bytes = jb >= 0 ? kKvBytes : 0u;
+      const int valid = U.n - key_a;
+      if (!a_is_v || valid >= kSub) {
         if (lane == 0) {
-          mbar_arrive_expect_tx(&sm.bar_full[r], kKvBytes);
-          for (int c = 0; c < kBoxes; ++c)
-            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, is_v ? &tv : &tk, &sm.bar_full[r], 64 * c, U.g, key0, U.b);
+          mbar_arrive_expect_tx(&sm.bar_full[r], kKvBytes + b_bytes);
+          load_kv(sm.ring[r][0], a_is_v ? &tv : &tk, &sm.bar_full[r], key_a, U);
+          if (jb >= 0) load_kv(sm.ring[r][1], &tk, &sm.bar_full[r], key_b, U);
         }
       } else {
         // Last, partial value sub-tile: rows >= n may hold any bit pattern and
@@ -271,19 +281,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         // shared memory before the MMA reads the tile.
         if (lane == 0) {
           mbar_arrive_expect_tx(&sm.bar_vtmp, kKvBytes);
-          for (int c = 0; c < kBoxes; ++c)
-            tma_load_4d(sm.ring[r] + c * kKvBoxBytes, &tv, &sm.bar_vtmp, 64 * c, U.g, key0, U.b);
+          load_kv(sm.ring[r][0], &tv, &sm.bar_vtmp, key_a, U);
         }
         ++vtmp;
         if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err)) return false;
         const int zrows = kSub - valid;
         for (int c = 0; c < kBoxes; ++c) {
-          uint4* base = reinterpret_cast<uint4*>(sm.ring[r] + c * kKvBoxBytes + valid * 128);
+          uint4* base = reinterpret_cast<uint4*>(sm.ring[r][0] + c * kKvBoxBytes + valid * 128);
           for (int e = lane; e < zrows * 8; e += 32) base[e] = make_uint4(0u, 0u, 0u, 0u);
         }
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.bar_full[r]);
+        if (lane == 0) {
+          if (jb >= 0) {
+            mbar_arrive_expect_tx(&sm.bar_full[r], b_bytes);
+            load_kv(sm.ring[r][1], &tk, &sm.bar_full[r], key_b, U);
+          } else {
+            mbar_arrive(&sm.bar_full[r]);
+          }
+        }
       }
       ++fills;
       return true;
@@ -293,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (U.nkv == 0) continue;
       // The unit's first key tiles need only ring slots: start them before
       // the query tiles, which wait for the previous unit's last score MMAs.
-      ok = fill(U, 0, false) && (U.nkv < 2 || fill(U, 1, false));
+      ok = fill(U, 0, false, U.nkv >= 2 ? 1 : -1);
       for (int i = 0; i < 2 && ok; ++i) {
         if (!U.run[i]) continue;
         // The slot's previous query tile is free once its last score MMA has run.
@@ -306,9 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++q_loads[i];
       }
       if (!ok) break;
-      for (int j = 0; ok && j < U.nkv; ++j) {
-        ok = fill(U, j, true) && (j + 2 >= U.nkv || fill(U, j + 2, false));
-      }
+      for (int j = 0; ok && j < U.nkv; ++j) ok = fill(U, j, true, j + 2 < U.nkv ? j + 2 : -1);
     }
     // Teardown: let every copy this warp issued land before the block exits.
     if (lane == 0) {
@@ -338,8 +352,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t q_addr = smem_u32(sm.q[i]);
       const uint32_t s_tmem = tmem + 256 * i;
       // S_i(j) -> buffer b: Q_i [128 x D] times K sub-tile [64 x D]^T.
-      auto issue_s = [&](int b, int r) {
-        const uint32_t kaddr = smem_u32(sm.ring[r]);
+      auto issue_s = [&](int b, const uint8_t* ktile) {
+        const uint32_t kaddr = smem_u32(ktile);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t qoff = (kk / 4) * kQBoxBytes + (kk % 4) * 32;
@@ -352,8 +366,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // O_i (+)= P_i(j) [128 x 64, tensor memory] times V sub-tile [64 x D].
       // Only the unit's last two PVs signal their completion (bar_pvm, bar_o):
       // for the others, the completion of the score MMA issued after them does.
-      auto issue_pv = [&](int b, int r, bool acc, uint64_t* done) {
-        const uint32_t vaddr = smem_u32(sm.ring[r]);
+      auto issue_pv = [&](int b, const uint8_t* vtile, bool acc, uint64_t* done) {
+        const uint32_t vaddr = smem_u32(vtile);
 #pragma unroll
         for (int kk = 0; kk < kSub / 16; ++kk) {
           mma_ts_elect(s_tmem + 128, s_tmem + kSub * b + kk * 8, sdesc_sw128(vaddr + kk * 16 * 128, kKvBoxBytes, 1024),
@@ -381,19 +395,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = warp_wait(&sm.bar_q[i], q_loads & 1, abort, p.err);
           ++q_loads;
         }
-        // Prologue: S(0) and S(1) into buffers 0 and 1.
-        for (int j = 0; ok && j < 2 && j < U.nkv; ++j, ++f) {
-          if (!wait_fill(f)) { ok = false; break; }
+        // Prologue: S(0) and S(1) into buffers 0 and 1 from the entry [K_0 | K_1].
+        {
+          const int fe = f++;
+          if (!wait_fill(fe)) { ok = false; break; }
           if (run) {
             tc_fence_after();
-            issue_s(j, f % kRing);
-            if (j == U.nkv - 1) mma_commit_elect(&sm.bar_qfree[i]);
+            issue_s(0, sm.ring[fe % kRing][0]);
+            if (U.nkv == 1) mma_commit_elect(&sm.bar_qfree[i]);
+            if (U.nkv >= 2) {
+              issue_s(1, sm.ring[fe % kRing][1]);
+              if (U.nkv == 2) mma_commit_elect(&sm.bar_qfree[i]);
+            }
           }
-          release(f, run);
+          release(fe, run);
         }
+        // Step j: PV(j) from the entry's V_j, then S(j + 2) from its K_{j+2}.
         for (int j = 0; ok && j < U.nkv; ++j) {
-          const int fv = f++;
-          if (!wait_fill(fv)) { ok = false; break; }
+          const int fe = f++;
+          if (!wait_fill(fe)) { ok = false; break; }
           if (run) {
             // O_i of this slot's previous unit must have been read out before PV(0) overwrites it.
             if (j == 0 && units_run > 0 && !warp_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err)) {
@@ -403,20 +423,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!warp_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
             ++p_seen;
             tc_fence_after();
-            issue_pv(j & 1, fv % kRing, j > 0,
+            issue_pv(j & 1, sm.ring[fe % kRing][0], j > 0,
                      j == U.nkv - 1 ? &sm.bar_o[i] : (j == U.nkv - 2 ? &sm.bar_pvm[i] : nullptr));
-          }
-          release(fv, run);
-          if (j + 2 < U.nkv) {
-            const int fk = f++;
-            if (!wait_fill(fk)) { ok = false; break; }
-            if (run) {
-              tc_fence_after();
-              issue_s(j & 1, fk % kRing);
+            if (j + 2 < U.nkv) {
+              issue_s(j & 1, sm.ring[fe % kRing][1]);
               if (j + 2 == U.nkv - 1) mma_commit_elect(&sm.bar_qfree[i]);
             }
-            release(fk, run);
           }
+          release(fe, run);
         }
         if (run) ++units_run;
       }
