@@ -887,7 +887,7 @@ def run_ours(args, rank, world):
     # The other workloads first: the projection GEMM below draws enough power
     # to leave the clocks under the power cap for a while after it.
     by_workload = {}
-    for name in [x for x in args.workloads.split(",") if x and not args.batch]:
+    for name in [x for x in args.workloads.split(",") if x and x != "none" and not args.batch]:
         by_workload[name] = measure_workload_kernels(Bn, name, d, peaks)
     lmhead_info = measure_lmhead(args, w, Bn, peaks) if args.lmhead_d > 0 else None
     e2e_lm = None if (args.no_e2e or args.lmhead_d <= 0) else measure_e2e_lmhead(args, Bn, w, world, d)
@@ -1009,7 +1009,7 @@ def main():
                     help="separate: dlm_vocab_confidence then dlm_refine_update (the faster of the two on "
                          "the 32 x 512 workload); fused: both in one launch (dlm_refine_step)")
     ap.add_argument("--workloads", default="c2_single_512,c4_long_2048,c5_heavy_4step",
-                    help="other workloads whose three kernels are also timed one by one (comma list; '' to skip)")
+                    help="other workloads whose three kernels are also timed one by one (comma list; none to skip)")
     ap.add_argument("--lmhead-d", type=int, default=2048,
                     help="also time the vocabulary projection fused with the reduction at this width (0: skip)")
     ap.add_argument("--attn-mask", default="full", choices=["full", "block_causal", "block_local"],

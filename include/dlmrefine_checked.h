@@ -21,6 +21,20 @@ extern "C" {
  */
 int dlm_checked_fill_static_scratch(int32_t byte_value);
 
+/*
+ * Sets the budget of every bounded wait in the attention and fused
+ * projection kernels launched afterwards by this library (default 2e9 ns;
+ * 100 .. 2e9 accepted, DLM_ERR_ARG otherwise). With a budget of a few hundred
+ * ns the waits of a real pipeline run out: the kernel records
+ * DLM_DEVERR_TIMEOUT, lets the copies and MMAs it issued land, frees its
+ * tensor memory and returns, leaving its outputs undefined. Calls made after
+ * setting the budget back to 2e9 are unaffected. A checked build times every
+ * wait, also one that completes at its first try, against the GPU's global
+ * timer, whose resolution is about a microsecond: waits shorter than that may
+ * not run out.
+ */
+int dlm_checked_set_wait_budget(int64_t budget_ns);
+
 #ifdef __cplusplus
 }
 #endif

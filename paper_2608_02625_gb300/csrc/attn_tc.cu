@@ -110,6 +110,7 @@ struct TcParams {
   int64_t so0, so1, so2;
   float scale_log2;
   int* err;
+  uint64_t wait_ns;  // budget of each bounded wait
 };
 
 struct Unit {
@@ -186,8 +187,9 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
 // producer and the MMA issuers walk the same order.
 
 // Warp-uniform bounded wait: true only if every lane saw the phase complete.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
-  bool ok = mbar_wait(bar, parity, abort, err);
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err,
+                                          uint64_t budget_ns) {
+  bool ok = mbar_wait_for(bar, parity, abort, err, budget_ns);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -264,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     auto fill = [&](const Unit& U, int ja, bool a_is_v, int jb) -> bool {
       const int r = fills % kRing;
-      if (fills >= kRing && !warp_wait(&sm.bar_empty[r], ((fills / kRing) - 1) & 1, abort, p.err)) return false;
+      if (fills >= kRing && !warp_wait(&sm.bar_empty[r], ((fills / kRing) - 1) & 1, abort, p.err, p.wait_ns)) return false;
       const int key_a = (kMasked ? U.kt(ja) : ja) * kSub;
       const int key_b = jb >= 0 ? (kMasked ? U.kt(jb) : jb) * kSub : 0;
       const uint32_t b_bytes = jb >= 0 ? kKvBytes : 0u;
@@ -284,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           load_kv(sm.ring[r][0], &tv, &sm.bar_vtmp, key_a, U);
         }
         ++vtmp;
-        if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err)) return false;
+        if (!warp_wait(&sm.bar_vtmp, (vtmp - 1) & 1, abort, p.err, p.wait_ns)) return false;
         const int zrows = kSub - valid;
         for (int c = 0; c < kBoxes; ++c) {
           uint4* base = reinterpret_cast<uint4*>(sm.ring[r][0] + c * kKvBoxBytes + valid * 128);
@@ -313,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < 2 && ok; ++i) {
         if (!U.run[i]) continue;
         // The slot's previous query tile is free once its last score MMA has run.
-        if (q_loads[i] > 0 && !warp_wait(&sm.bar_qfree[i], (q_loads[i] - 1) & 1, abort, p.err)) { ok = false; break; }
+        if (q_loads[i] > 0 && !warp_wait(&sm.bar_qfree[i], (q_loads[i] - 1) & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
         if (lane == 0) {
           mbar_arrive_expect_tx(&sm.bar_q[i], kQBytes);
           for (int c = 0; c < kBoxes; ++c)
@@ -376,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (done) mma_commit_elect(done);
       };
       auto wait_fill = [&](int f) -> bool {
-        return warp_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err);
+        return warp_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err, p.wait_ns);
       };
       auto release = [&](int f, bool issued) {
         if (issued) mma_commit_elect(&sm.bar_empty[f % kRing]);
@@ -392,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (U.nkv == 0) continue;
         const bool run = U.run[i];
         if (run) {
-          ok = warp_wait(&sm.bar_q[i], q_loads & 1, abort, p.err);
+          ok = warp_wait(&sm.bar_q[i], q_loads & 1, abort, p.err, p.wait_ns);
           ++q_loads;
         }
         // Prologue: S(0) and S(1) into buffers 0 and 1 from the entry [K_0 | K_1].
@@ -416,11 +418,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!wait_fill(fe)) { ok = false; break; }
           if (run) {
             // O_i of this slot's previous unit must have been read out before PV(0) overwrites it.
-            if (j == 0 && units_run > 0 && !warp_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err)) {
+            if (j == 0 && units_run > 0 && !warp_wait(&sm.bar_ofree[i], (units_run - 1) & 1, abort, p.err, p.wait_ns)) {
               ok = false;
               break;
             }
-            if (!warp_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err)) { ok = false; break; }
+            if (!warp_wait(&sm.bar_p[i][p_seen & 1], (p_seen >> 1) & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
             ++p_seen;
             tc_fence_after();
             issue_pv(j & 1, sm.ring[fe % kRing][0], j > 0,
@@ -479,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // bursts alternate instead of coinciding.
         uint64_t t0 = global_timer_ns();
         while (*reinterpret_cast<volatile int*>(&sm.unit_flag) < unit_seq) {
-          if (global_timer_ns() - t0 > kWaitBudgetNs || *abort) { *abort = 1; ok = false; break; }
+          if (global_timer_ns() - t0 > p.wait_ns || *abort) { *abort = 1; ok = false; break; }
         }
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       }
@@ -494,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (s_ahead[b]) {
           s_ahead[b] = false;
         } else {
-          if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err)) { ok = false; break; }
+          if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
           ++s_seen[b];
         }
         tc_fence_after();
@@ -536,11 +538,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             // for PV(j-1)'s own barrier, then rescale.
             if (j + 1 < U.nkv) {
               const int bn = b ^ 1;
-              if (!warp_wait(&sm.bar_s[i][bn], s_seen[bn] & 1, abort, p.err)) { ok = false; break; }
+              if (!warp_wait(&sm.bar_s[i][bn], s_seen[bn] & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
               ++s_seen[bn];
               s_ahead[bn] = true;
             } else {
-              if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err)) { ok = false; break; }
+              if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
               ++pvm_seen;
               pvm_done = true;
             }
@@ -591,10 +593,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // The unit's last two PVs (the next-to-last one only if not consumed above).
       if (ok && U.nkv >= 2 && !pvm_done) {
-        if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err)) ok = false;
+        if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err, p.wait_ns)) ok = false;
         ++pvm_seen;
       }
-      if (!ok || !warp_wait(&sm.bar_o[i], units_run & 1, abort, p.err)) { ok = false; break; }
+      if (!ok || !warp_wait(&sm.bar_o[i], units_run & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
       ++units_run;
       // Epilogue: read O_i out of tensor memory, hand the columns back to the
       // MMA warp, then normalise, convert to bf16, stage 32 rows x 32 columns
@@ -725,6 +727,7 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   p.so2 = a.so[2];
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(D));
   p.err = device_error_word();
+  p.wait_ns = wait_budget_ns();
   const size_t smem = sizeof(Smem<D>) + 1024;
   cudaError_t attr_err = cudaFuncSetAttribute(attn_tc_kernel<D, kMasked>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(smem));

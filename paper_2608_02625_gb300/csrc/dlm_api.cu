@@ -4,6 +4,7 @@
 // negative dlm_status before any launch when something is wrong. Values that
 // live in device memory (lengths) are clamped by the kernels, which record it
 // in the per-device error word read by dlm_get_device_error.
+#include <atomic>
 #include <cstdarg>
 #include <cmath>
 #include <cstdint>
@@ -26,6 +27,8 @@ thread_local char t_last_error[512] = "";
 constexpr int kMaxDevices = 64;
 std::mutex g_err_mu;
 int* g_err_addr[kMaxDevices] = {};
+
+std::atomic<uint64_t> g_wait_budget_ns{dlm::kDefaultWaitBudgetNs};
 
 int64_t elem_size(int dtype) {
   switch (dtype) {
@@ -118,6 +121,8 @@ int fail(int status, const char* fmt, ...) {
 void clear_error() { t_last_error[0] = '\0'; }
 
 cudaStream_t current_stream() { return t_stream; }
+
+uint64_t wait_budget_ns() { return g_wait_budget_ns.load(std::memory_order_relaxed); }
 
 int* device_error_word() {
   int dev = 0;
@@ -684,6 +689,14 @@ extern "C" int dlm_checked_fill_static_scratch(int32_t byte_value) {
   if (const int st = dlm::static_step_scratch(&scratch)) return st;
   const cudaError_t e = cudaMemsetAsync(scratch, byte_value, sizeof(g_dlm_step_scratch), t_stream);
   if (e != cudaSuccess) return fail(DLM_ERR_CUDA, "filling the static step scratch: %s", cudaGetErrorString(e));
+  return DLM_OK;
+}
+
+extern "C" int dlm_checked_set_wait_budget(int64_t budget_ns) {
+  t_last_error[0] = '\0';
+  if (budget_ns < 100 || budget_ns > static_cast<int64_t>(dlm::kDefaultWaitBudgetNs))
+    return dlm::fail(DLM_ERR_ARG, "budget_ns %lld outside [100, 2e9]", static_cast<long long>(budget_ns));
+  g_wait_budget_ns.store(static_cast<uint64_t>(budget_ns), std::memory_order_relaxed);
   return DLM_OK;
 }
 #endif  // DLM_CHECK_BOUNDS

@@ -30,6 +30,15 @@ __device__ __forceinline__ void set_device_error(int* err, int bits) {
   if (err) atomicOr(err, bits);
 }
 
+// Builds compiled with DLM_CHECK_BOUNDS check the inputs' value contracts in
+// the kernels (NaN or all -inf logit rows, token ids out of range) and report
+// a violation as DLM_DEVERR_INPUT; the default build does not pay for it.
+#ifdef DLM_CHECK_BOUNDS
+constexpr bool kCheckBounds = true;
+#else
+constexpr bool kCheckBounds = false;
+#endif
+
 // ----------------------------------------------------------------- mbarrier
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -97,6 +106,23 @@ constexpr uint64_t kWaitBudgetNs = 2000000000ull;  // 2 s
 // and DLM_DEVERR_TIMEOUT in the error word.
 __device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort, int* err,
                                               uint64_t budget_ns) {
+  if constexpr (kCheckBounds) {
+    // Checked builds time every wait, also one whose phase completes within
+    // the first try (mbarrier.try_wait suspends the thread in hardware for a
+    // while, so short waits never reach the loop below): a budget of a few
+    // hundred ns then makes the waits of a real pipeline run out, in tests.
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 1;; ++it) {
+      const bool done = mbar_try_wait(bar, parity);
+      if (global_timer_ns() - t0 > budget_ns) {
+        *abort = 1;
+        set_device_error(err, DLM_DEVERR_TIMEOUT);
+        return false;
+      }
+      if (done) return true;
+      if ((it & 63u) == 0u && *abort) return false;
+    }
+  }
   if (mbar_try_wait(bar, parity)) return true;
   uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
@@ -321,15 +347,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N, bo
   return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn_major ? 1u : 0u) << 15) |
          ((b_mn_major ? 1u : 0u) << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
-
-// Builds compiled with DLM_CHECK_BOUNDS check the inputs' value contracts in
-// the kernels (NaN or all -inf logit rows, token ids out of range) and report
-// a violation as DLM_DEVERR_INPUT; the default build does not pay for it.
-#ifdef DLM_CHECK_BOUNDS
-constexpr bool kCheckBounds = true;
-#else
-constexpr bool kCheckBounds = false;
-#endif
 
 // ----------------------------------------------------------------- math
 

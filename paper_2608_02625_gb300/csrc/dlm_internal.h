@@ -12,6 +12,12 @@ namespace dlm {
 // Device address of the error word of the current device (set up once per device).
 int* device_error_word();
 
+// Budget of each bounded wait in the pipelined kernels (ns): 2 s, which no
+// legitimate wait inside one launch approaches. Only DLM_CHECK_BOUNDS builds
+// can change it (dlm_checked_set_wait_budget), to make waits run out in tests.
+constexpr uint64_t kDefaultWaitBudgetNs = 2000000000ull;
+uint64_t wait_budget_ns();
+
 // Device address of dlm_refine_step_static's scratch array on the current
 // device (set up on first use; a status, with *out untouched, on failure).
 int static_step_scratch(int32_t** out);

@@ -69,6 +69,7 @@ struct LmParams {
   int* part_idx;
   float* part_s;
   int* err;
+  uint64_t wait_ns;  // budget of each bounded wait
 };
 
 struct Item {
@@ -84,8 +85,9 @@ __device__ __forceinline__ Item item_at(const LmParams& p, int item) {
   return it;
 }
 
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err) {
-  bool ok = mbar_wait(bar, parity, abort, err);
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err,
+                                          uint64_t budget_ns) {
+  bool ok = mbar_wait_for(bar, parity, abort, err, budget_ns);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -134,7 +136,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int vt = it.t0; ok && vt < it.t1; ++vt) {
         for (int kb = 0; kb < kblocks; ++kb, ++fill) {
           const int st = fill % kStages;
-          if (fill >= kStages && !warp_wait(&sm.empty[st], ((fill / kStages) - 1) & 1, abort, p.err)) {
+          if (fill >= kStages && !warp_wait(&sm.empty[st], ((fill / kStages) - 1) & 1, abort, p.err, p.wait_ns)) {
             ok = false;
             break;
           }
@@ -167,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int vt = it.t0; ok && vt < it.t1; ++vt, ++tile) {
           const int acc = tile & 1;
           // The accumulator's previous tile (tile - 2) must have been read out.
-          if (tile >= 2 && !warp_wait(&sm.acc_empty[acc], ((tile >> 1) - 1) & 1, abort, p.err)) {
+          if (tile >= 2 && !warp_wait(&sm.acc_empty[acc], ((tile >> 1) - 1) & 1, abort, p.err, p.wait_ns)) {
             ok = false;
             break;
           }
@@ -175,7 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t d_tmem = tmem + acc * kBN;
           for (int kb = 0; kb < kblocks; ++kb, ++fill) {
             const int st = fill % kStages;
-            if (!warp_wait(&sm.full[st], (fill / kStages) & 1, abort, p.err)) {
+            if (!warp_wait(&sm.full[st], (fill / kStages) & 1, abort, p.err, p.wait_ns)) {
               ok = false;
               break;
             }
@@ -209,7 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int idx = 0;
       for (int vt = it.t0; vt < it.t1; ++vt, ++tile) {
         const int acc = tile & 1;
-        if (!warp_wait(&sm.acc_full[acc], (tile >> 1) & 1, abort, p.err)) {
+        if (!warp_wait(&sm.acc_full[acc], (tile >> 1) & 1, abort, p.err, p.wait_ns)) {
           ok = false;
           break;
         }
@@ -371,6 +373,7 @@ int launch_lmhead(const LmArgs& a, cudaStream_t stream) {
   p.part_idx = reinterpret_cast<int*>(ws + static_cast<int64_t>(p.splits) * a.N);
   p.part_s = ws + 2 * static_cast<int64_t>(p.splits) * a.N;
   p.err = device_error_word();
+  p.wait_ns = wait_budget_ns();
   CUtensorMap mh, mw;
   int st;
   if ((st = make_map_2d(&mh, a.hidden, a.N, p.d, a.s_hidden, kBM)) != DLM_OK) return st;

@@ -329,10 +329,13 @@ def test_checked_build_exports_its_test_hooks(tmp_path):
     checked = ctypes.CDLL(str(tmp_path / "libdlmrefine.so"))
     default = ctypes.CDLL(os.path.join(PKG, "libdlmrefine.so"))
     hooks = declared_functions("dlmrefine_checked.h")
-    assert hooks == ["dlm_checked_fill_static_scratch"]
+    assert hooks == ["dlm_checked_fill_static_scratch", "dlm_checked_set_wait_budget"]
     for n in declared_functions("dlmrefine.h") + hooks:
         assert hasattr(checked, n), f"checked build does not export {n}"
     for n in hooks:
         assert not hasattr(default, n), f"default build exports the test hook {n}"
     checked.dlm_checked_fill_static_scratch.argtypes = [ctypes.c_int32]
     assert checked.dlm_checked_fill_static_scratch(256) == -6
+    checked.dlm_checked_set_wait_budget.argtypes = [ctypes.c_int64]
+    assert checked.dlm_checked_set_wait_budget(99) == -6 and checked.dlm_checked_set_wait_budget(2000000001) == -6
+    assert checked.dlm_checked_set_wait_budget(2000000000) == 0

@@ -126,3 +126,84 @@ def test_static_step_clears_poisoned_scratch(tmp_path):
             assert torch.equal(x, y), f"call {call + 1}: {name} differs from the workspace call"
     bits = ctypes.c_int32(0)
     assert checked.dlm_get_device_error(ctypes.byref(bits), 1) == 0 and bits.value == 0
+
+
+@pytest.mark.gpu
+def test_real_pipelines_time_out_and_recover(tmp_path):
+    """With a wait budget of 300 ns (checked build) the pipelined kernels' waits
+    on their TMA loads and MMAs run out: attention and the fused projection
+    return, record DLM_DEVERR_TIMEOUT and tear down (in-flight copies and MMAs
+    drained, tensor memory freed). With the budget back at 2 s the same calls
+    are correct and leave the error word clean."""
+    import time
+
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_02625_gb300 import binding as Bn
+    from paper_2608_02625_gb300 import build
+    build.build(check_bounds=True, out_dir=str(tmp_path))
+    lib = ctypes.CDLL(str(tmp_path / "libdlmrefine.so"))
+    lib.dlm_checked_set_wait_budget.argtypes = [ctypes.c_int64]
+    lib.dlm_lmhead_workspace_bytes.argtypes = [ctypes.c_int64]
+    lib.dlm_lmhead_workspace_bytes.restype = ctypes.c_size_t
+    d = torch.device("cuda", 0)
+    torch.cuda.set_device(d)
+    assert lib.dlm_set_stream(ctypes.c_void_p(torch.cuda.current_stream(d).cuda_stream)) == 0
+
+    def bits():
+        b = ctypes.c_int32(0)
+        assert lib.dlm_get_device_error(ctypes.byref(b), 1) == 0
+        return b.value
+
+    def descs(ts):
+        return [ctypes.byref(Bn.describe(t)) for t in ts]
+
+    g = torch.Generator().manual_seed(12)
+    q = torch.randn(1, 256, 4, 128, generator=g).to(torch.bfloat16)
+    k = torch.randn(1, 256, 2, 128, generator=g).to(torch.bfloat16)
+    v = torch.randn(1, 256, 2, 128, generator=g).to(torch.bfloat16)
+    sl = torch.tensor([250], dtype=torch.int32)
+    # d = 2048: the projection's epilogue waits for 32 k-blocks of MMAs per
+    # tile (microseconds), longer than the resolution of the GPU's global
+    # timer, which the waits read.
+    hid = torch.randn(256, 2048, generator=g).to(torch.bfloat16)
+    wt = (torch.randn(4096, 2048, generator=g) / 45).to(torch.bfloat16)
+    qd, kd, vd, sld, hd, wd = (t.to(d) for t in (q, k, v, sl, hid, wt))
+    out = torch.empty_like(qd)
+    am = torch.empty(256, dtype=torch.int32, device=d)
+    cf = torch.empty(256, dtype=torch.float32, device=d)
+    ls = torch.empty(256, dtype=torch.float32, device=d)
+    nws = lib.dlm_lmhead_workspace_bytes(256)
+    ws = torch.empty(nws, dtype=torch.uint8, device=d)
+
+    def attn():
+        return lib.dlm_bidir_attn(*descs((qd, kd, vd, sld, out)))
+
+    def lmhead():
+        return lib.dlm_lmhead_confidence(*descs((hd, wd, am, cf, ls)), ctypes.c_void_p(ws.data_ptr()),
+                                         ctypes.c_size_t(nws))
+
+    assert bits() == 0
+    assert lib.dlm_checked_set_wait_budget(300) == 0
+    try:
+        for name, call in (("attention", attn), ("projection", lmhead)):
+            t0 = time.perf_counter()
+            assert call() == 0
+            torch.cuda.synchronize()
+            assert time.perf_counter() - t0 < 5.0, name
+            assert bits() & 0x2, f"{name}: no DLM_DEVERR_TIMEOUT with a 300 ns budget"
+    finally:
+        assert lib.dlm_checked_set_wait_budget(2000000000) == 0
+    assert attn() == 0 and lmhead() == 0
+    torch.cuda.synchronize()
+    assert bits() == 0
+    ref = oracle.bidir_attn(q.float().numpy(), k.float().numpy(), v.float().numpy(), [250])
+    assert np.abs(out.float().cpu().numpy() - ref).max() <= 2e-2
+    lg = oracle.lm_head_logits(hid.float().numpy(), wt.float().numpy())
+    r_am, _, r_ls = oracle.vocab_confidence(lg)
+    top2 = np.sort(lg, axis=1)[:, -2:]
+    clear = top2[:, 1] - top2[:, 0] > 1e-3
+    assert np.array_equal(am.cpu().numpy()[clear], r_am[clear])
+    assert np.abs(ls.cpu().numpy() - r_ls).max() <= 1e-3
