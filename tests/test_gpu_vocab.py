@@ -42,7 +42,8 @@ def test_workload_all_rows(name):
 
 @pytest.mark.parametrize("name", ["c3_batch32_512", "c4_long_2048", "c5_heavy_4step"])
 def test_workload_sampled_rows(name):
-    """Full-size launch; the oracle recomputes a spread sample of rows one by one."""
+    """Full-size launch; the oracle recomputes ~180 rows one by one (random,
+    and at the edges of waves of CTAs and of sequences)."""
     w = workloads.get(name)
     from paper_2608_02625_gb300 import synth_gpu
     tok, msk = w.initial_state()
@@ -51,7 +52,12 @@ def test_workload_sampled_rows(name):
     x = synth_gpu.logits(w, 0, dev(), t_tok, t_msk)
     am, cf, ls = gpu_vocab(x)
     rng = np.random.default_rng(5)
-    rows = np.unique(np.concatenate([[0, w.N - 1], rng.integers(0, w.N, 40)]))
+    # 160 random rows, plus rows at the edges of waves of resident CTAs (4 per
+    # SM on 152 SMs) and of sequences.
+    wave = 4 * 152
+    edges = [r for k in range(1, 4) for r in (k * wave - 1, k * wave) if r < w.N]
+    seq_edges = [r for b in (0, 1, w.B // 2, w.B - 1) for r in (b * w.L, b * w.L + w.L - 1)]
+    rows = np.unique(np.concatenate([[0, w.N - 1], edges, seq_edges, rng.integers(0, w.N, 160)]))
     ref = oracle.vocab_confidence(host_logit_rows(w, 0, rows, tok.reshape(-1)[rows], msk.reshape(-1)[rows]))
     check_vocab(am[rows], cf[rows], ls[rows], *ref, where=name)
     del x
