@@ -411,6 +411,40 @@ def measure_loop(args, w, Bn, q, k, v, out, logits, tok0, msk0, params, seqlen, 
                     "graph: CUDA events around one launch; host-driven: wall clock, one n_edits read-back per pass"}
 
 
+def measure_fused_step(Bn, w, logits, tok, msk, params, stream, per_kernel, reps=20):
+    """The vocabulary reduction and the update in one launch (dlm_refine_step)
+    on the step's own resident buffers, against the two separate launches
+    timed in the step (CUDA events around `reps` back-to-back launches)."""
+    import torch
+    d = logits.device
+    am = torch.empty((w.B, w.L), dtype=torch.int32, device=d)
+    cf = torch.empty((w.B, w.L), dtype=torch.float32, device=d)
+    ls = torch.empty((w.B, w.L), dtype=torch.float32, device=d)
+    nt, nm = torch.empty_like(tok), torch.empty_like(msk)
+    ne = torch.empty(w.B, dtype=torch.int32, device=d)
+    ws = torch.zeros(Bn.dlm_refine_step_workspace_bytes(w.B) // 4, dtype=torch.int32, device=d)
+
+    def run():
+        Bn.dlm_refine_step(logits, tok, msk, params, am, cf, ls, nt, nm, ne, ws)
+
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if Bn.device_error(clear=True):
+        raise RuntimeError("device error word set during the fused-step measurement")
+    ms = e0.elapsed_time(e1) / reps
+    sep = per_kernel["vocab"] + per_kernel["update"]
+    return {"ms": ms, "ms_separate_vocab_plus_update": sep, "ratio_fused_over_separate": ms / sep,
+            "note": "dlm_refine_step (one launch: the CTA finishing a sequence's last row runs its update) on the "
+                    "step's buffers; the step itself uses the separate launches, the faster of the two here"}
+
+
 def measure_lmhead(args, w, Bn, peaks, reps=10):
     """The vocabulary projection fused with the reduction (dlm_lmhead_confidence)
     on the workload's N rows and V tokens at width d = --lmhead-d, against the
@@ -894,6 +928,7 @@ def run_ours(args, rank, world):
     loop_info = None
     if args.loop_steps > 0:
         loop_info = measure_loop(args, w, Bn, q, k, v, out, logits, tok, msk, params, seqlen, stream)
+    fused_info = None if fused else measure_fused_step(Bn, w, logits, tok, msk, params, stream, per_kernel)
 
     attn_flops = w.attn_flops(mask_mode, args.block)
     vocab_bytes = w.vocab_bytes()
@@ -947,6 +982,7 @@ def run_ours(args, rank, world):
         "attn_mask": args.attn_mask if not mask_mode else f"{args.attn_mask} (block {args.block})",
         "e2e": e2e,
         "loop": loop_info,
+        "fused_step": fused_info,
         "lmhead": lmhead_info,
         "e2e_lmhead": e2e_lm,
         "kernels_by_workload": by_workload,
