@@ -113,11 +113,17 @@ struct TcParams {
   uint64_t wait_ns;  // budget of each bounded wait
 };
 
+// A value per slot, read with a select: the slot index comes from the warp,
+// and an array indexed by it would live in local memory.
+struct Pair {
+  int v0, v1;
+  __device__ __forceinline__ int operator[](int i) const { return i ? v1 : v0; }
+};
+
 struct Unit {
   int b, g, n, p, nkv;  // nkv: 64-key sub-tiles visited
   int ka, kgap;         // sub-tile j of the unit is key sub-tile kt(j) = j < ka ? j : j + kgap
-  int head[2], row0[2];
-  bool active[2], run[2];
+  Pair head, row0, active, run;
   __device__ __forceinline__ int kt(int j) const { return j < ka ? j : j + kgap; }
 };
 
@@ -135,13 +141,16 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
   }
   U.n = n;
   const int ntiles = p.G * p.mtiles;
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const int t = 2 * u + i;
-    U.active[i] = t < ntiles;
-    U.head[i] = U.g * p.G + (U.active[i] ? t % p.G : 0);
-    U.row0[i] = (U.active[i] ? t / p.G : 0) * kTile;
-    U.run[i] = U.active[i] && U.row0[i] < n;
+  {
+    const int t0 = 2 * u, t1 = 2 * u + 1;
+    U.active.v0 = t0 < ntiles;
+    U.active.v1 = t1 < ntiles;
+    U.head.v0 = U.g * p.G + (U.active.v0 ? t0 % p.G : 0);
+    U.head.v1 = U.g * p.G + (U.active.v1 ? t1 % p.G : 0);
+    U.row0.v0 = (U.active.v0 ? t0 / p.G : 0) * kTile;
+    U.row0.v1 = (U.active.v1 ? t1 / p.G : 0) * kTile;
+    U.run.v0 = U.active.v0 && U.row0.v0 < n;
+    U.run.v1 = U.active.v1 && U.row0.v1 < n;
   }
   U.p = 0;
   U.ka = U.nkv = (U.run[0] || U.run[1]) ? (n + kSub - 1) / kSub : 0;
@@ -249,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kProducerWarp) {
     // ================================================================ TMA producer
-    int q_loads[2] = {0, 0};   // query loads per slot (= bar_q / bar_qfree phases)
+    int q_loads0 = 0, q_loads1 = 0;  // query loads per slot (= bar_q / bar_qfree phases)
     int fills = 0;             // ring fills issued; slot fills % kRing, phase (fills / kRing) & 1
     int vtmp = 0;              // private partial-V fills
     bool ok = true;
@@ -315,21 +324,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = 0; i < 2 && ok; ++i) {
         if (!U.run[i]) continue;
         // The slot's previous query tile is free once its last score MMA has run.
-        if (q_loads[i] > 0 && !warp_wait(&sm.bar_qfree[i], (q_loads[i] - 1) & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
+        const int ql = i ? q_loads1 : q_loads0;
+        if (ql > 0 && !warp_wait(&sm.bar_qfree[i], (ql - 1) & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
         if (lane == 0) {
           mbar_arrive_expect_tx(&sm.bar_q[i], kQBytes);
           for (int c = 0; c < kBoxes; ++c)
             tma_load_4d(sm.q[i] + c * kQBoxBytes, &tq, &sm.bar_q[i], 64 * c, U.head[i], U.row0[i], U.b);
         }
-        ++q_loads[i];
+        if (i) ++q_loads1; else ++q_loads0;
       }
       if (!ok) break;
       for (int j = 0; ok && j < U.nkv; ++j) ok = fill(U, j, true, j + 2 < U.nkv ? j + 2 : -1);
     }
     // Teardown: let every copy this warp issued land before the block exits.
     if (lane == 0) {
-      for (int i = 0; i < 2; ++i)
-        if (q_loads[i]) mbar_drain(&sm.bar_q[i], (q_loads[i] - 1) & 1);
+      if (q_loads0) mbar_drain(&sm.bar_q[0], (q_loads0 - 1) & 1);
+      if (q_loads1) mbar_drain(&sm.bar_q[1], (q_loads1 - 1) & 1);
       if (vtmp) mbar_drain(&sm.bar_vtmp, (vtmp - 1) & 1);
       for (int r = 0; r < kRing; ++r) {
         const int n_r = fills > r ? (fills - r + kRing - 1) / kRing : 0;  // fills of slot r
