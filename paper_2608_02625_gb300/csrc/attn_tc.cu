@@ -101,8 +101,31 @@ struct Smem {
   int unit_flag;   // units whose first slot-0 hand-off happened
 };
 
+// Division by a divisor fixed at launch as a multiply-high and a shift
+// (Granlund and Montgomery, "Division by invariant integers using
+// multiplication", PLDI 1994): for 0 <= n < 2^31 and d >= 1, with
+// l = ceil(log2 d) and m = floor(2^(32 + l) / d) - 2^32 + 1,
+// n / d = (umulhi(n, m) + n) >> l (the sum stays below 2^32).
+struct FastDiv {
+  uint32_t d, m, l;
+  __device__ __forceinline__ int div(int n) const {
+    const uint32_t u = static_cast<uint32_t>(n);
+    return static_cast<int>((__umulhi(u, m) + u) >> l);
+  }
+};
+
+FastDiv make_fastdiv(int d) {
+  FastDiv f;
+  f.d = static_cast<uint32_t>(d);
+  f.l = 0;
+  while ((1ull << f.l) < f.d) ++f.l;
+  f.m = static_cast<uint32_t>((1ull << (32 + f.l)) / f.d - (1ull << 32) + 1);
+  return f;
+}
+
 struct TcParams {
   int B, L, Hq, Hkv, G, mtiles, units_per_bg, units;
+  FastDiv div_upb, div_hkv, div_g;  // by units_per_bg, Hkv, G
   int mask_mode, block;
   const int32_t* seq_lens;
   const int32_t* prompt_lens;
@@ -130,10 +153,10 @@ struct Unit {
 template <bool kMasked>
 __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
   Unit U;
-  const int bg = unit / p.units_per_bg;
-  const int u = unit % p.units_per_bg;
-  U.b = bg / p.Hkv;
-  U.g = bg % p.Hkv;
+  const int bg = p.div_upb.div(unit);
+  const int u = unit - bg * p.units_per_bg;
+  U.b = p.div_hkv.div(bg);
+  U.g = bg - U.b * p.Hkv;
   int n = p.seq_lens ? p.seq_lens[U.b] : p.L;
   if (n < 0 || n > p.L) {
     if (threadIdx.x == 0) set_device_error(p.err, DLM_DEVERR_LENGTH);
@@ -145,10 +168,11 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
     const int t0 = 2 * u, t1 = 2 * u + 1;
     U.active.v0 = t0 < ntiles;
     U.active.v1 = t1 < ntiles;
-    U.head.v0 = U.g * p.G + (U.active.v0 ? t0 % p.G : 0);
-    U.head.v1 = U.g * p.G + (U.active.v1 ? t1 % p.G : 0);
-    U.row0.v0 = (U.active.v0 ? t0 / p.G : 0) * kTile;
-    U.row0.v1 = (U.active.v1 ? t1 / p.G : 0) * kTile;
+    const int r0 = p.div_g.div(t0), r1 = p.div_g.div(t1);
+    U.head.v0 = U.g * p.G + (U.active.v0 ? t0 - r0 * p.G : 0);
+    U.head.v1 = U.g * p.G + (U.active.v1 ? t1 - r1 * p.G : 0);
+    U.row0.v0 = (U.active.v0 ? r0 : 0) * kTile;
+    U.row0.v1 = (U.active.v1 ? r1 : 0) * kTile;
     U.run.v0 = U.active.v0 && U.row0.v0 < n;
     U.run.v1 = U.active.v1 && U.row0.v1 < n;
   }
@@ -459,14 +483,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = static_cast<uint32_t>(qw * 32) << 16;
     const uint32_t slot_addr = tmem + lane_base + 256 * i;
     const uint32_t o_addr = slot_addr + 128;
-    int s_seen[2] = {0, 0};  // bar_s phases consumed per buffer
+    uint32_t s_par = 0;      // bit b: parity of the next bar_s[i][b] phase
     int unit_seq = 0;
     // PV completion: S(j) is issued after PV(j-2) and S(j+1) after PV(j-1)
     // (one issuer, in order), so waiting for a score buffer also waits for the
     // PVs before it. Only the unit's last two PVs have barriers of their own
     // (bar_pvm, bar_o), each consumed once per unit; their next phases need
     // hand-offs of the next unit, so they cannot run two phases ahead.
-    bool s_ahead[2] = {false, false};  // next phase of bar_s[i][b] already consumed
+    uint32_t s_ahead = 0;    // bit b: the next phase of bar_s[i][b] already consumed
     int hand = 0;       // hand-offs so far: hand-off n on bar_p[i][n % 2]
     int pvm_seen = 0;   // bar_pvm phases consumed
     int units_run = 0;  // bar_o phases consumed
@@ -503,11 +527,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < U.nkv; ++j) {
         const int b = j & 1;
         const uint32_t s_addr = slot_addr + kSub * b;
-        if (s_ahead[b]) {
-          s_ahead[b] = false;
+        if ((s_ahead >> b) & 1u) {
+          s_ahead &= ~(1u << b);
         } else {
-          if (!warp_wait(&sm.bar_s[i][b], s_seen[b] & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
-          ++s_seen[b];
+          if (!warp_wait(&sm.bar_s[i][b], (s_par >> b) & 1u, abort, p.err, p.wait_ns)) { ok = false; break; }
+          s_par ^= 1u << b;
         }
         tc_fence_after();
         uint32_t sr[kSub];
@@ -548,9 +572,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             // for PV(j-1)'s own barrier, then rescale.
             if (j + 1 < U.nkv) {
               const int bn = b ^ 1;
-              if (!warp_wait(&sm.bar_s[i][bn], s_seen[bn] & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
-              ++s_seen[bn];
-              s_ahead[bn] = true;
+              if (!warp_wait(&sm.bar_s[i][bn], (s_par >> bn) & 1u, abort, p.err, p.wait_ns)) { ok = false; break; }
+              s_par ^= 1u << bn;
+              s_ahead |= 1u << bn;
             } else {
               if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
               ++pvm_seen;
@@ -616,43 +640,47 @@ __global__ void __launch_bounds__(kThreads, 1)
       // row r at position e ^ ((r / 2) % 4)), which makes the warp's stores
       // free of shared-memory bank conflicts.
       tc_fence_after();
-      uint32_t ov[D];
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) tmem_ld32(o_addr + 32 * c, *reinterpret_cast<uint32_t(*)[32]>(&ov[32 * c]));
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&sm.bar_ofree[i]);
       const bool valid_row = row < U.n;
       const float inv = valid_row ? 1.0f / l : 0.f;
       const int wrow0 = U.row0[i] + 32 * qw;
-      if (wrow0 < p.L) {
+      const bool store = wrow0 < p.L;
+      if (store) {
         if (lane == 0) bulk_wait_read<0>();  // staging buffers of the previous unit are free
         __syncwarp();
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint8_t* buf = sm.stage[warp][c & 1];
-          if (c >= 2) {
-            if (lane == 0) bulk_wait_read<1>();
-            __syncwarp();
-          }
-          uint8_t* dstrow = buf + lane * 64;
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            uint32_t w[4];
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const int col = 32 * c + 8 * e + 2 * h;
-              w[h] = valid_row ? pack_bf16x2(__uint_as_float(ov[col]) * inv, __uint_as_float(ov[col + 1]) * inv)
-                               : 0u;
-            }
-            *reinterpret_cast<uint4*>(dstrow + ((e ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-          }
-          fence_proxy_async_smem();
+      }
+      // One 32-column chunk of O at a time (a compact loop: this code runs
+      // once per unit); the columns go back to the MMA warp after the last.
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t ov[32];
+        tmem_ld32(o_addr + 32 * c, ov);
+        tmem_wait_ld();
+        if (c == D / 32 - 1) {
+          tc_fence_before();
+          mbar_arrive(&sm.bar_ofree[i]);
+        }
+        if (!store) continue;
+        uint8_t* buf = sm.stage[warp][c & 1];
+        if (c >= 2) {
+          if (lane == 0) bulk_wait_read<1>();
           __syncwarp();
-          if (lane == 0) {
-            tma_store_4d(&to, buf, 32 * c, U.head[i], wrow0, U.b);
-            bulk_commit();
+        }
+        uint8_t* dstrow = buf + lane * 64;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          uint32_t w[4];
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const int col = 8 * e + 2 * h;
+            w[h] = valid_row ? pack_bf16x2(__uint_as_float(ov[col]) * inv, __uint_as_float(ov[col + 1]) * inv) : 0u;
           }
+          *reinterpret_cast<uint4*>(dstrow + ((e ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_4d(&to, buf, 32 * c, U.head[i], wrow0, U.b);
+          bulk_commit();
         }
       }
     }
@@ -723,6 +751,9 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   p.G = a.Hq / a.Hkv;
   p.mtiles = (a.L + kTile - 1) / kTile;
   p.units_per_bg = (p.G * p.mtiles + 1) / 2;
+  p.div_upb = make_fastdiv(p.units_per_bg);
+  p.div_hkv = make_fastdiv(p.Hkv);
+  p.div_g = make_fastdiv(p.G);
   const long long units = static_cast<long long>(a.B) * a.Hkv * p.units_per_bg;
   if (units == 0) return DLM_OK;
   if (units > 0x7FFFFFFFLL) return fail(DLM_ERR_SHAPE, "too many attention work units");
