@@ -642,6 +642,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const bool valid_row = row < U.n;
       const float inv = valid_row ? 1.0f / l : 0.f;
+      const float2 inv2 = make_float2(inv, inv);
+      // Rows >= n are written as zeros whatever O holds there (a NaN times
+      // zero would not be zero).
+      const uint32_t vmask = valid_row ? 0xFFFFFFFFu : 0u;
       const int wrow0 = U.row0[i] + 32 * qw;
       const bool store = wrow0 < p.L;
       if (store) {
@@ -672,7 +676,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
             const int col = 8 * e + 2 * h;
-            w[h] = valid_row ? pack_bf16x2(__uint_as_float(ov[col]) * inv, __uint_as_float(ov[col + 1]) * inv) : 0u;
+            const float2 x = fmul2(make_float2(__uint_as_float(ov[col]), __uint_as_float(ov[col + 1])), inv2);
+            w[h] = pack_bf16x2(x.x, x.y) & vmask;
           }
           *reinterpret_cast<uint4*>(dstrow + ((e ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
