@@ -219,6 +219,15 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
 // holds the two tiles one step of an issuer reads: PV(j) and S(j + 2). The
 // producer and the MMA issuers walk the same order.
 
+// Bits [a - key0, b - key0) of a 64-bit word, clamped to [0, 64): the keys
+// a <= key < b of the sub-tile that starts at key0.
+__device__ __forceinline__ uint64_t key_bits(int key0, int a, int b) {
+  const int lo = max(a - key0, 0), hi = min(b - key0, 64);
+  if (hi <= lo) return 0ull;
+  const uint64_t below_hi = hi >= 64 ? ~0ull : (1ull << hi) - 1ull;
+  return below_hi & ~((1ull << lo) - 1ull);  // lo < hi <= 64
+}
+
 // Warp-uniform bounded wait: true only if every lane saw the phase complete.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err,
                                           uint64_t budget_ns) {
@@ -543,10 +552,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kSub; ++c) sv[c] = __uint_as_float(sr[c]);
         const int key0 = (kMasked ? U.kt(j) : j) * kSub;
         if (!(key0 + kSub <= kr.hi1 || (kMasked && key0 >= kr.lo2 && key0 + kSub <= kr.hi2))) {
+          // The row's keys in this sub-tile, [0, hi1) and [lo2, hi2), as bits;
+          // one bit test per score.
+          const uint64_t allow = key_bits(key0, 0, kr.hi1) | (kMasked ? key_bits(key0, kr.lo2, kr.hi2) : 0ull);
+          const uint32_t alo = static_cast<uint32_t>(allow), ahi = static_cast<uint32_t>(allow >> 32);
 #pragma unroll
           for (int c = 0; c < kSub; ++c) {
-            const int key = key0 + c;
-            if (!(key < kr.hi1 || (kMasked && key >= kr.lo2 && key < kr.hi2))) sv[c] = -INFINITY;
+            if (!(((c < 32 ? alo : ahi) >> (c & 31)) & 1u)) sv[c] = -INFINITY;
           }
         }
         float mx0 = sv[0], mx1 = sv[1], mx2 = sv[2], mx3 = sv[3];
