@@ -369,6 +369,17 @@ int dlm_set_stream(void* stream);
 /* The stream currently set for this thread. */
 void* dlm_get_stream(void);
 
+/* Work granularity of the BF16 attention kernels (dlm_bidir_attn,
+ * dlm_attn_masked) for later calls on this thread; no effect on results.
+ * A work unit is one or two 128-row query tiles of one sequence and key/value
+ * head, run by one CTA. tiles = 2: two tiles per unit, which share each
+ * key/value tile the CTA loads (the faster choice once there are at least as
+ * many pairs of tiles as SMs); 1: one tile per unit (a single short sequence:
+ * every tile runs at once); 0: automatic, the default (1 when the pairs of
+ * tiles are fewer than the SMs, else 2). Returns DLM_ERR_ARG for any other
+ * value, leaving the setting unchanged. */
+int dlm_set_attn_tiles_per_unit(int tiles);
+
 /* Static description of a status code. */
 const char* dlm_status_string(int status);
 /* Message for the most recent failure on this thread ("" if none). */

@@ -61,7 +61,7 @@ def _load():
     lib.dlm_refine_step_workspace_bytes.restype = ctypes.c_size_t
     for f in ("dlm_bidir_attn", "dlm_attn_masked", "dlm_vocab_confidence", "dlm_refine_update", "dlm_refine_step",
               "dlm_refine_step_static", "dlm_token_prob", "dlm_refine_update_ranked", "dlm_lmhead_confidence",
-              "dlm_set_stream",
+              "dlm_set_stream", "dlm_set_attn_tiles_per_unit",
               "dlm_version", "dlm_get_device_error"):
         getattr(lib, f).restype = ctypes.c_int
     lib.dlm_loop_begin.argtypes = [ctypes.c_void_p]
@@ -74,6 +74,7 @@ def _load():
     lib.dlm_selftest_wait_timeout.argtypes = [ctypes.c_int64]
     lib.dlm_selftest_wait_timeout.restype = ctypes.c_int
     lib.dlm_set_stream.argtypes = [ctypes.c_void_p]
+    lib.dlm_set_attn_tiles_per_unit.argtypes = [ctypes.c_int]
     lib.dlm_get_stream.restype = ctypes.c_void_p
     lib.dlm_status_string.restype = ctypes.c_char_p
     lib.dlm_status_string.argtypes = [ctypes.c_int]
@@ -317,6 +318,11 @@ def dlm_loop_end(n_edits: torch.Tensor, max_steps: int, steps_out: torch.Tensor)
 def dlm_loop_cancel():
     """Ends an unfinished recording on this thread, keeping nothing."""
     _check(lib.dlm_loop_cancel())
+
+
+def dlm_set_attn_tiles_per_unit(tiles: int):
+    """Query tiles per attention work unit on this thread: 0 automatic, 1 or 2."""
+    _check(lib.dlm_set_attn_tiles_per_unit(int(tiles)))
 
 
 def dlm_selftest_wait_timeout(budget_ns: int, device: int | None = None):

@@ -9,9 +9,11 @@
 // Work unit: two 128-row query tiles ("slots") that read the same key/value
 // head of the same sequence (two query heads of one GQA group, or two row
 // blocks of one head), so each key/value tile staged in shared memory feeds
-// both. The kernel is persistent: one CTA per SM walks units blockIdx.x,
-// blockIdx.x + gridDim.x, ...; the next unit's query tiles load as soon as the
-// slot's last score MMA has run, and its first score MMAs overlap the epilogue.
+// both. With fewer pairs of tiles than SMs (a single short sequence) a unit
+// is one tile in slot 0, slot 1 idles, and every tile runs at once. The kernel
+// is persistent: one CTA per SM walks units blockIdx.x, blockIdx.x +
+// gridDim.x, ...; the next unit's query tiles load as soon as the slot's last
+// score MMA has run, and its first score MMAs overlap the epilogue.
 //
 // Keys are processed in 64-key sub-tiles so that each slot's scores can be
 // double-buffered in tensor memory: the tensor core computes S(j+1) while the
@@ -125,6 +127,7 @@ FastDiv make_fastdiv(int d) {
 
 struct TcParams {
   int B, L, Hq, Hkv, G, mtiles, units_per_bg, units;
+  int tpu;  // query tiles per unit: 2 (both slots), 1 (slot 0 only: few tiles)
   FastDiv div_upb, div_hkv, div_g;  // by units_per_bg, Hkv, G
   int mask_mode, block;
   const int32_t* seq_lens;
@@ -165,7 +168,7 @@ __device__ __forceinline__ Unit decode_unit(const TcParams& p, int unit) {
   U.n = n;
   const int ntiles = p.G * p.mtiles;
   {
-    const int t0 = 2 * u, t1 = 2 * u + 1;
+    const int t0 = p.tpu * u, t1 = p.tpu == 2 ? t0 + 1 : ntiles;
     U.active.v0 = t0 < ntiles;
     U.active.v1 = t1 < ntiles;
     const int r0 = p.div_g.div(t0), r1 = p.div_g.div(t1);
@@ -767,7 +770,16 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   p.Hkv = a.Hkv;
   p.G = a.Hq / a.Hkv;
   p.mtiles = (a.L + kTile - 1) / kTile;
-  p.units_per_bg = (p.G * p.mtiles + 1) / 2;
+  // Two query tiles per work unit, one in each slot; when that leaves SMs
+  // idle (a single short sequence), one tile per unit, so that every tile
+  // runs at once.
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long pairs = static_cast<long long>(a.B) * a.Hkv * ((p.G * p.mtiles + 1) / 2);
+  const int forced = attn_tiles_per_unit();
+  p.tpu = forced ? forced : (pairs < sms ? 1 : 2);
+  p.units_per_bg = (p.G * p.mtiles + p.tpu - 1) / p.tpu;
   p.div_upb = make_fastdiv(p.units_per_bg);
   p.div_hkv = make_fastdiv(p.Hkv);
   p.div_g = make_fastdiv(p.G);
@@ -790,9 +802,6 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   cudaError_t attr_err = cudaFuncSetAttribute(attn_tc_kernel<D, kMasked>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               static_cast<int>(smem));
   if (attr_err != cudaSuccess) return fail(DLM_ERR_CUDA, "attn smem attribute: %s", cudaGetErrorString(attr_err));
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = static_cast<int>(units < sms ? units : sms);
   attn_tc_kernel<D, kMasked><<<grid, kThreads, smem, stream>>>(mq, mk, mv, mo, p);
   cudaError_t e = cudaGetLastError();

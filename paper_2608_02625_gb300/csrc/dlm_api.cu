@@ -22,6 +22,7 @@ namespace {
 __device__ int g_dlm_device_error;
 
 thread_local cudaStream_t t_stream = nullptr;
+thread_local int t_attn_tpu = 0;  // query tiles per attention work unit (0: automatic)
 thread_local char t_last_error[512] = "";
 
 constexpr int kMaxDevices = 64;
@@ -124,6 +125,8 @@ cudaStream_t current_stream() { return t_stream; }
 
 uint64_t wait_budget_ns() { return g_wait_budget_ns.load(std::memory_order_relaxed); }
 
+int attn_tiles_per_unit() { return t_attn_tpu; }
+
 int* device_error_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
@@ -176,6 +179,12 @@ int dlm_set_stream(void* stream) {
 }
 
 void* dlm_get_stream(void) { return t_stream; }
+
+int dlm_set_attn_tiles_per_unit(int tiles) {
+  if (tiles < 0 || tiles > 2) return dlm::fail(DLM_ERR_ARG, "dlm_set_attn_tiles_per_unit: %d is not 0, 1 or 2", tiles);
+  t_attn_tpu = tiles;
+  return DLM_OK;
+}
 
 int dlm_get_device_error(int32_t* bits, int clear) {
   if (!bits) return dlm::fail(DLM_ERR_NULL, "dlm_get_device_error: bits is NULL");

@@ -17,6 +17,8 @@ int* device_error_word();
 // can change it (dlm_checked_set_wait_budget), to make waits run out in tests.
 constexpr uint64_t kDefaultWaitBudgetNs = 2000000000ull;
 uint64_t wait_budget_ns();
+// Query tiles per attention work unit set on this thread (0: automatic).
+int attn_tiles_per_unit();
 
 // Device address of dlm_refine_step_static's scratch array on the current
 // device (set up on first use; a status, with *out untouched, on failure).

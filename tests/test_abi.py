@@ -339,3 +339,12 @@ def test_checked_build_exports_its_test_hooks(tmp_path):
     checked.dlm_checked_set_wait_budget.argtypes = [ctypes.c_int64]
     assert checked.dlm_checked_set_wait_budget(99) == -6 and checked.dlm_checked_set_wait_budget(2000000001) == -6
     assert checked.dlm_checked_set_wait_budget(2000000000) == 0
+
+
+def test_attn_tiles_per_unit_setting():
+    from paper_2608_02625_gb300.binding import lib
+    for bad in (-1, 3, 1 << 20):
+        assert lib.dlm_set_attn_tiles_per_unit(bad) == -6
+        assert b"dlm_set_attn_tiles_per_unit" in lib.dlm_last_error()
+    for ok in (1, 2, 0):
+        assert lib.dlm_set_attn_tiles_per_unit(ok) == 0

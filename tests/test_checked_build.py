@@ -186,6 +186,11 @@ def test_real_pipelines_time_out_and_recover(tmp_path):
                                          ctypes.c_size_t(nws))
 
     assert bits() == 0
+    # Two query tiles per attention unit: the second slot's start waits for
+    # the first slot's first hand-off, a wait of microseconds, longer than the
+    # resolution of the global timer the waits read. With one tile per unit
+    # (the automatic choice at this size) every wait can end within one tick.
+    assert lib.dlm_set_attn_tiles_per_unit(2) == 0
     assert lib.dlm_checked_set_wait_budget(300) == 0
     try:
         for name, call in (("attention", attn), ("projection", lmhead)):
@@ -196,6 +201,7 @@ def test_real_pipelines_time_out_and_recover(tmp_path):
             assert bits() & 0x2, f"{name}: no DLM_DEVERR_TIMEOUT with a 300 ns budget"
     finally:
         assert lib.dlm_checked_set_wait_budget(2000000000) == 0
+        assert lib.dlm_set_attn_tiles_per_unit(0) == 0
     assert attn() == 0 and lmhead() == 0
     torch.cuda.synchronize()
     assert bits() == 0

@@ -92,8 +92,14 @@ def run_case(B, L, Hq, Hkv, D, seq_lens, sigma, dtype="bf16", seed=0):
     (3, 256, 4, 2, 64, [256, 1, 129]),        # head_dim 64
     (6, 260, 2, 1, 128, [0, 1, 127, 128, 129, 260]),  # edge lengths
 ])
-def test_bf16_cases(B, L, Hq, Hkv, D, sl, sigma):
-    run_case(B, L, Hq, Hkv, D, sl, sigma, "bf16", seed=B * L + Hq)
+@pytest.mark.parametrize("tiles", [0, 1, 2])
+def test_bf16_cases(B, L, Hq, Hkv, D, sl, sigma, tiles):
+    from paper_2608_02625_gb300 import binding as Bn
+    Bn.dlm_set_attn_tiles_per_unit(tiles)
+    try:
+        run_case(B, L, Hq, Hkv, D, sl, sigma, "bf16", seed=B * L + Hq)
+    finally:
+        Bn.dlm_set_attn_tiles_per_unit(0)
 
 
 @pytest.mark.parametrize("B,L,Hq,Hkv,D,sl", [(1, 128, 4, 2, 64, [128]), (2, 200, 4, 1, 128, [200, 77])])
@@ -207,3 +213,33 @@ def test_workload_full_size(name, pairs):
             g = (h * w.Hkv) // w.Hq
             ref = oracle.bidir_attn(hq[None, :, h:h + 1], hk[None, :, g:g + 1], hv[None, :, g:g + 1], [n[b]])
             compare(g_out[b:b + 1, :, h:h + 1], ref, [n[b]], tol, where=f"{name} b={b} h={h}")
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("B,L,Hq,Hkv,D,sl,pl", [
+    (2, 384, 6, 2, 128, [384, 257], [64, 100]),   # odd group size: pairs cross heads and rows
+    (1, 512, 32, 4, 128, [512], [160]),           # one sequence of the paper's length
+    (3, 256, 4, 2, 64, [256, 1, 129], [0, 0, 64]),  # head_dim 64, edge lengths
+])
+def test_tiles_per_unit_bit_identical(B, L, Hq, Hkv, D, sl, pl, mode):
+    """One or two query tiles per work unit changes only which CTA slot runs a
+    tile: every tile's arithmetic is the same, so the outputs are bit-identical."""
+    from paper_2608_02625_gb300 import binding as Bn
+    q, k, v = (t.to(dev()) for t in rand_qkv(B, L, Hq, Hkv, D, 1.0, "bf16", 17 + mode))
+    n = torch.tensor(sl, dtype=torch.int32, device=dev())
+    p = torch.tensor(pl, dtype=torch.int32, device=dev())
+    outs = []
+    for tiles in (1, 2):
+        out = torch.full(q.shape, float("nan"), dtype=q.dtype, device=dev())
+        Bn.dlm_set_attn_tiles_per_unit(tiles)
+        try:
+            if mode == 0:
+                Bn.dlm_bidir_attn(q, k, v, n, out)
+            else:
+                Bn.dlm_attn_masked(q, k, v, n, p, mode, 64, out)
+        finally:
+            Bn.dlm_set_attn_tiles_per_unit(0)
+        torch.cuda.synchronize()
+        assert Bn.device_error(clear=True) == 0
+        outs.append(out)
+    assert torch.equal(outs[0], outs[1])
