@@ -14,6 +14,9 @@
 //           given probability of the kept token elsewhere);
 //   pass 3  remask keys below the k-th key, and the lowest-index positions
 //           whose key equals it (an ordered block scan), up to k_b in total.
+// Responses of at most 4 keys per thread compute each key once, in pass 1,
+// and keep it in shared memory for passes 2 and 3; longer ones re-read the
+// predictions in each pass.
 // Integer work and exact fp32 compares only: results are bit-exact.
 // Used by the stand-alone update kernel (update.cu) and by the fused
 // vocabulary + update kernel (vocab.cu), whose last row block of a sequence
@@ -30,9 +33,11 @@ namespace dlm {
 
 template <int kThreads>
 struct UpdateShared {
+  static constexpr int kKeyCap = 4 * kThreads;  // response positions whose keys are kept here
   int hist[256];
   int warp_sums[kThreads / 32];
   int sel_digit, sel_before;
+  uint32_t keys[kKeyCap];  // ranking key of response position p + j (responses of at most kKeyCap)
 };
 
 // Order-preserving map of an fp32 value to uint32 (smaller value -> smaller
@@ -114,20 +119,30 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
   };
 
   // ---- pass 1: copy / commit / edit (read and write of position i by one
-  // thread, so new_* may alias tokens/mask)
+  // thread, so new_* may alias tokens/mask). Responses of at most kKeyCap
+  // positions also keep each position's ranking key in shared memory, so
+  // that the selection below reads the predictions once.
+  const bool cached = r <= UpdateShared<kThreads>::kKeyCap;
+  bool saw_nan = false;
   int edits = 0;
   for (int i = tid; i < L; i += kThreads) {
     int t = tok[i];
     uint8_t m = msk[i];
     if (i >= p && i < n) {
-      int pred = load_pred<kFresh>(am + i);
+      const int pred = load_pred<kFresh>(am + i);
+      const float c = load_pred<kFresh>(cf + i);
       if (m) {
         t = pred;
-      } else if (pred != t && load_pred<kFresh>(cf + i) >= a.edit_threshold) {
+      } else if (pred != t && c >= a.edit_threshold) {
         t = pred;
         ++edits;
       }
       m = 0;
+      if (cached) {
+        const float v = (tp && t != pred) ? tp[i] : c;
+        saw_nan |= is_nan_bits(__float_as_uint(v));
+        sh.keys[i - p] = conf_key(v);
+      }
     }
     ntok[i] = t;
     nmsk[i] = m;
@@ -156,9 +171,15 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
   }
 
   // ---- pass 2: radix select of the k-th smallest key (1-based rank `need`)
+  // The key of response position i (pass 1's copy when cached).
+  auto key_of = [&](int i) -> uint32_t {
+    if (cached) return sh.keys[i - p];
+    const float c = rank_value(i);
+    saw_nan |= is_nan_bits(__float_as_uint(c));
+    return conf_key(c);
+  };
   uint32_t prefix = 0, pmask = 0;
   int need = static_cast<int>(k);
-  bool saw_nan = false;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = tid; i < 256; i += kThreads) sh.hist[i] = 0;
     __syncthreads();
@@ -167,9 +188,7 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
       bool active = false;
       uint32_t digit = 0;
       if (i < n) {
-        const float c = rank_value(i);
-        if (shift == 24 && is_nan_bits(__float_as_uint(c))) saw_nan = true;
-        uint32_t key = conf_key(c);
+        const uint32_t key = key_of(i);
         if ((key & pmask) == prefix) {
           active = true;
           digit = (key >> shift) & 0xFFu;
@@ -219,7 +238,7 @@ __device__ void refine_sequence(const UpdateArgs& a, int b, int* err, UpdateShar
   int taken = 0;
   for (int base = p; base < n; base += kThreads) {
     int i = base + tid;
-    uint32_t key = i < n ? conf_key(rank_value(i)) : 0xFFFFFFFFu;
+    uint32_t key = i < n ? key_of(i) : 0xFFFFFFFFu;
     bool eq = i < n && key == kth;
     int total;
     int incl = block_inclusive_scan<kThreads>(eq ? 1 : 0, sh.warp_sums, &total);
