@@ -192,3 +192,34 @@ def test_empty_batch_needs_no_workspace():
                        z(0, 4), z(0, 4, dt=torch.float32), z(0, 4, dt=torch.float32), z(0, 4),
                        z(0, 4, dt=torch.uint8), z(0), z(0))
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("r", [1023, 1024, 1025])
+def test_key_cache_boundary(r):
+    """The fused step's update at the capacity of its shared-memory key cache
+    (four keys per thread of the 256-thread vocabulary block: 1024 response
+    positions) and one past it: equal to the separate update on the same
+    predictions, and to the oracle under the decision-margin protocol."""
+    from paper_2608_02625_gb300 import binding as Bn
+    rng = np.random.default_rng(9000 + r)
+    d = dev()
+    B, L, V = 2, r + 30, 64
+    case = P.random_update_case(rng, B=B, L=L, V=V, ties=False)
+    case["prompt_lens"] = np.array([0, 30])
+    case["seq_lens"] = case["prompt_lens"] + r
+    x = random_logits(rng, B * L, V, "bf16", ties=True)
+    logits = torch.from_numpy(x).to(torch.bfloat16).to(d)
+    tok = torch.from_numpy(case["tokens"]).to(d)
+    msk = torch.from_numpy(case["mask"]).to(d)
+    prompt = torch.from_numpy(case["prompt_lens"].astype(np.int32)).to(d)
+    seqlen = torch.from_numpy(case["seq_lens"].astype(np.int32)).to(d)
+    params = Bn.RefineParams(0.5, -1, 0.1, case["V"], prompt, seqlen)
+    ws = torch.zeros(B, dtype=torch.int32, device=d)
+    fz = run_fused(logits, tok, msk, params, ws)
+    names = ("tokens", "mask", "n_edits")
+    assert_equal_outputs(fz[3:], gpu_update_from(fz, tok, msk, params), names, f"r={r} vs update call")
+    ref_v = oracle.vocab_confidence(x)
+    pn = dict(edit_threshold=0.5, remask_k=-1, remask_frac=0.1, mask_id=case["V"],
+              prompt_lens=case["prompt_lens"], seq_lens=case["seq_lens"])
+    oracle_update_parity(fz, case["tokens"], case["mask"], pn, ref_v, f"r={r} oracle update")
+

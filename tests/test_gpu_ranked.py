@@ -165,3 +165,22 @@ def test_workload_rows_chain():
     gpu = pr.cpu().numpy()[rows].astype(np.float64)
     lse_err = np.abs(ls.cpu().numpy()[rows].astype(np.float64) - lse_ref) + 1e-7
     assert np.all(np.abs(gpu - ref) <= (CONF_RTOL + 2 * lse_err) * ref + 1e-37)
+
+
+@pytest.mark.parametrize("r", [2047, 2048, 2049])
+def test_key_cache_boundary(r):
+    """The ranked update at the capacity of the shared-memory key cache (2048
+    response positions) and one past it: keys of both kinds, with ties."""
+    rng = np.random.default_rng(5000 + r)
+    L = r + 40
+    case = P.random_update_case(rng, B=3, L=L, V=40, ties=True)
+    case["prompt_lens"] = np.array([0, 17, 40])
+    case["seq_lens"] = case["prompt_lens"] + r
+    tp = rng.choice(np.array([0.0, 0.25, 0.5], dtype=np.float32), (3, L))
+    ref = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"], edit_threshold=0.25,
+                               remask_k=-1, remask_frac=0.1, mask_id=case["V"], prompt_lens=case["prompt_lens"],
+                               seq_lens=case["seq_lens"], tok_prob=tp)
+    gpu = run_ranked(case["tokens"], case["mask"], case["argmax"], case["conf"], tp, tau=0.25, k=-1, frac=0.1,
+                     mask_id=case["V"], prompt=case["prompt_lens"], seqlen=case["seq_lens"])
+    same(gpu, ref, f"r={r}")
+

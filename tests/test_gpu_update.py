@@ -126,3 +126,23 @@ def test_editable_window(lo, hi):
         out = np.r_[0:wlo[b], whi[b]:L]
         assert np.array_equal(gpu[0][b, out], case["tokens"][b, out])
         assert np.array_equal(gpu[1][b, out], case["mask"][b, out])
+
+
+@pytest.mark.parametrize("r", [2047, 2048, 2049])
+def test_key_cache_boundary(r):
+    """Responses at the capacity of the shared-memory key cache (four keys per
+    thread of the 512-thread update: 2048 positions) and one past it, heavy
+    ties included, against the oracle."""
+    rng = np.random.default_rng(r)
+    L = r + 40
+    case = P.random_update_case(rng, B=3, L=L, V=40, ties=True)
+    case["prompt_lens"] = np.array([0, 17, 40])
+    case["seq_lens"] = case["prompt_lens"] + r
+    for k, frac in ((-1, 0.1), (r // 3, 0.0), (1, 0.0)):
+        ref = oracle.refine_update(case["tokens"], case["mask"], case["argmax"], case["conf"], edit_threshold=0.25,
+                                   remask_k=k, remask_frac=frac, mask_id=case["V"], prompt_lens=case["prompt_lens"],
+                                   seq_lens=case["seq_lens"])
+        gpu = run_gpu(case["tokens"], case["mask"], case["argmax"], case["conf"], tau=0.25, k=k, frac=frac,
+                      mask_id=case["V"], prompt=case["prompt_lens"], seqlen=case["seq_lens"])
+        assert_same(gpu, ref, f"r={r} k={k}")
+
