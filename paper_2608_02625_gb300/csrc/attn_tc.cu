@@ -27,8 +27,9 @@
 //              sub-tiles through a ring of four entries of two sub-tiles each,
 //              in the order the issuers consume them -- [K_0 | K_1], then
 //              [V_j | K_{j+2}] for each j -- so that each step of an issuer
-//              waits for one fill and releases one entry; an entry is
-//              released as soon as the MMAs that read it have completed
+//              waits for one fill; an entry is released, per slot, by the
+//              slot's softmax warps once they see the completion of the MMAs
+//              that read it (no tcgen05.commit for it in the issuer)
 //   warp 9     tensor-memory allocator; MMA issuer of slot 0 (one lane elected
 //              per instruction)
 //   warp 10    MMA issuer of slot 1
@@ -90,7 +91,7 @@ struct Smem {
   uint64_t bar_q[2];          // query tile of slot i landed          (TMA -> MMA)
   uint64_t bar_qfree[2];      // last score MMA of slot i completed   (MMA -> TMA)
   uint64_t bar_full[kRing];   // ring slot filled (V padding cleared)  (TMA -> MMA)
-  uint64_t bar_empty[kRing];  // ring slot read by its MMAs           (MMA -> TMA)
+  uint64_t bar_empty[kRing];  // ring slot read by its MMAs, per slot (softmax or idle issuer -> TMA)
   uint64_t bar_s[2][2];       // S_i buffer b ready                   (MMA -> softmax)
   uint64_t bar_p[2][2];       // hand-off n of slot i (P written, O rescaled) on bar_p[i][n % 2] (softmax -> MMA)
   uint64_t bar_pvm[2];        // the unit's next-to-last PV of slot i completed (MMA -> softmax)
@@ -272,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int r = 0; r < kRing; ++r) {
       mbar_init(&sm.bar_full[r], 1);
-      mbar_init(&sm.bar_empty[r], 2);  // one arrival per MMA issuer
+      mbar_init(&sm.bar_empty[r], 2);  // one release per slot
     }
     mbar_init(&sm.bar_vtmp, 1);
     mbar_init(&sm.bar_done[0], 1);
@@ -389,10 +390,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // streams do not wait on each other's hand-offs; each stream is ordered on
     // its own. All 32 lanes run the issue loop (waits are warp-uniform) and
     // one lane elected inside each instruction issues it: no branch around the
-    // MMAs, whose operands then stay in uniform registers. Both issuers arrive
-    // on every ring slot's release barrier: with tcgen05.commit after their
-    // MMAs read the slot, or with a plain arrive (after the fill landed) when
-    // their slot idles in a unit.
+    // MMAs, whose operands then stay in uniform registers. Every ring entry
+    // gets one release per slot: from the slot's softmax warps when the slot
+    // runs in the unit, else from its issuer with a plain arrive once the
+    // fill has landed.
     const int i = warp - kMmaWarp0;
     {
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, kSub, false, false);  // Q, K both K-major
@@ -426,9 +427,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto wait_fill = [&](int f) -> bool {
         return warp_wait(&sm.bar_full[f % kRing], (f / kRing) & 1, abort, p.err, p.wait_ns);
       };
+      // A running slot's entries are released by its softmax warps, which see
+      // the completion of the MMAs that read them (below); an idle slot
+      // releases each entry once its fill has landed.
       auto release = [&](int f, bool issued) {
-        if (issued) mma_commit_elect(&sm.bar_empty[f % kRing]);
-        else mbar_arrive_elect(&sm.bar_empty[f % kRing]);
+        if (!issued) mbar_arrive_elect(&sm.bar_empty[f % kRing]);
       };
       int q_loads = 0;    // bar_q phases consumed
       int units_run = 0;  // bar_ofree phases
@@ -496,6 +499,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t slot_addr = tmem + lane_base + 256 * i;
     const uint32_t o_addr = slot_addr + 128;
     uint32_t s_par = 0;      // bit b: parity of the next bar_s[i][b] phase
+    // Ring entries of the running unit: [K_0 | K_1] at f0, [V_j | K_{j+2}] at
+    // f0 + 1 + j. The MMAs of one issuer complete in order, so once S(x) has
+    // completed so have PV(x - 2) and S(x), the readers of entry x - 2: one
+    // thread per slot releases an entry when it sees that completion.
+    int f_next = 0;          // ring entries of the units walked so far
+    const bool rel_thread = t == 0;
     int unit_seq = 0;
     // PV completion: S(j) is issued after PV(j-2) and S(j+1) after PV(j-1)
     // (one issuer, in order), so waiting for a score buffer also waits for the
@@ -509,6 +518,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int unit = blockIdx.x; ok && unit < p.units; unit += gridDim.x) {
       const Unit U = decode_unit<kMasked>(p, unit);
+      const int f0 = f_next;
+      if (U.nkv > 0) f_next += U.nkv + 1;
       if (!U.active[i]) continue;
       const int row = U.row0[i] + t;
       if (!U.run[i]) {
@@ -536,6 +547,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool pvm_done = false;
       // This row's keys: [0, hi1) and [lo2, hi2).
       const KeyRanges kr = kMasked ? key_ranges(p.mask_mode, p.block, row, U.n, U.p) : KeyRanges{U.n, U.n, U.n};
+      // S(x) seen complete: release the entry it and PV(x - 2) read.
+      auto scores_seen = [&](int x) {
+        if (!rel_thread) return;
+        if (x >= 2) mbar_arrive(&sm.bar_empty[(f0 + x - 1) % kRing]);
+        else if (x == 1 || U.nkv == 1) mbar_arrive(&sm.bar_empty[f0 % kRing]);
+      };
       for (int j = 0; j < U.nkv; ++j) {
         const int b = j & 1;
         const uint32_t s_addr = slot_addr + kSub * b;
@@ -544,6 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           if (!warp_wait(&sm.bar_s[i][b], (s_par >> b) & 1u, abort, p.err, p.wait_ns)) { ok = false; break; }
           s_par ^= 1u << b;
+          scores_seen(j);
         }
         tc_fence_after();
         uint32_t sr[kSub];
@@ -590,10 +608,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (!warp_wait(&sm.bar_s[i][bn], (s_par >> bn) & 1u, abort, p.err, p.wait_ns)) { ok = false; break; }
               s_par ^= 1u << bn;
               s_ahead |= 1u << bn;
+              scores_seen(j + 1);
             } else {
               if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
               ++pvm_seen;
               pvm_done = true;
+              if (rel_thread) mbar_arrive(&sm.bar_empty[(f0 + U.nkv - 1) % kRing]);  // [V_{n-2}]
             }
             tc_fence_after();
 #pragma unroll 1
@@ -644,8 +664,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (ok && U.nkv >= 2 && !pvm_done) {
         if (!warp_wait(&sm.bar_pvm[i], pvm_seen & 1, abort, p.err, p.wait_ns)) ok = false;
         ++pvm_seen;
+        if (ok && rel_thread) mbar_arrive(&sm.bar_empty[(f0 + U.nkv - 1) % kRing]);  // [V_{n-2}]
       }
       if (!ok || !warp_wait(&sm.bar_o[i], units_run & 1, abort, p.err, p.wait_ns)) { ok = false; break; }
+      if (rel_thread) mbar_arrive(&sm.bar_empty[(f0 + U.nkv) % kRing]);  // [V_{n-1}]
       ++units_run;
       // Epilogue: read O_i out of tensor memory, hand the columns back to the
       // MMA warp, then normalise, convert to bf16, stage 32 rows x 32 columns
