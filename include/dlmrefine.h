@@ -373,11 +373,11 @@ void* dlm_get_stream(void);
  * dlm_attn_masked) for later calls on this thread; no effect on results.
  * A work unit is one or two 128-row query tiles of one sequence and key/value
  * head, run by one CTA. tiles = 2: two tiles per unit, which share each
- * key/value tile the CTA loads (the faster choice once there are at least as
- * many pairs of tiles as SMs); 1: one tile per unit (a single short sequence:
- * every tile runs at once); 0: automatic, the default (1 when the pairs of
- * tiles are fewer than the SMs, else 2). Returns DLM_ERR_ARG for any other
- * value, leaving the setting unchanged. */
+ * key/value tile the CTA loads (the faster choice unless every single tile
+ * fits on the SMs at once); 1: one tile per unit (a single short sequence:
+ * every tile runs at once); 0: automatic, the default (1 when twice the
+ * number of tile pairs is at most the SM count, else 2). Returns DLM_ERR_ARG
+ * for any other value, leaving the setting unchanged. */
 int dlm_set_attn_tiles_per_unit(int tiles);
 
 /* Static description of a status code. */

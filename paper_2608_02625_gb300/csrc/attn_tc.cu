@@ -9,8 +9,8 @@
 // Work unit: two 128-row query tiles ("slots") that read the same key/value
 // head of the same sequence (two query heads of one GQA group, or two row
 // blocks of one head), so each key/value tile staged in shared memory feeds
-// both. With fewer pairs of tiles than SMs (a single short sequence) a unit
-// is one tile in slot 0, slot 1 idles, and every tile runs at once. The kernel
+// both. When even single tiles all fit on the SMs at once (a single short
+// sequence) a unit is one tile in slot 0 and slot 1 idles. The kernel
 // is persistent: one CTA per SM walks units blockIdx.x, blockIdx.x +
 // gridDim.x, ...; the next unit's query tiles load as soon as the slot's last
 // score MMA has run, and its first score MMAs overlap the epilogue.
@@ -792,15 +792,17 @@ int launch_d(const AttnArgs& a, cudaStream_t stream) {
   p.Hkv = a.Hkv;
   p.G = a.Hq / a.Hkv;
   p.mtiles = (a.L + kTile - 1) / kTile;
-  // Two query tiles per work unit, one in each slot; when that leaves SMs
-  // idle (a single short sequence), one tile per unit, so that every tile
-  // runs at once.
+  // Two query tiles per work unit, one in each slot; one tile per unit only
+  // when every tile then runs at once (twice the pairs still fit on the SMs:
+  // a single short sequence). One-tile units take ~0.8 of a two-tile unit's
+  // time, so a second round of them costs more than the pairs' one round
+  // (measured at 1 x 512: 10.0 against 12.0 us; at 2 x 512: 17.2 against 12.8).
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const long long pairs = static_cast<long long>(a.B) * a.Hkv * ((p.G * p.mtiles + 1) / 2);
   const int forced = attn_tiles_per_unit();
-  p.tpu = forced ? forced : (pairs < sms ? 1 : 2);
+  p.tpu = forced ? forced : (2 * pairs <= sms ? 1 : 2);
   p.units_per_bg = (p.G * p.mtiles + p.tpu - 1) / p.tpu;
   p.div_upb = make_fastdiv(p.units_per_bg);
   p.div_hkv = make_fastdiv(p.Hkv);
