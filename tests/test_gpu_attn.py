@@ -243,3 +243,21 @@ def test_tiles_per_unit_bit_identical(B, L, Hq, Hkv, D, sl, pl, mode):
         assert Bn.device_error(clear=True) == 0
         outs.append(out)
     assert torch.equal(outs[0], outs[1])
+
+
+def test_workload_tiles_bit_identical():
+    """The whole 32 x 512 launch with one and with two query tiles per unit:
+    every (sequence, head) pair bit-identical whichever slot ran it."""
+    from paper_2608_02625_gb300 import binding as Bn, synth_gpu
+    w = workloads.get("c3_batch32_512")
+    q, k, v = synth_gpu.qkv(w, 0, dev())
+    n = w.seq_lens()
+    outs = []
+    for tiles in (1, 2):
+        Bn.dlm_set_attn_tiles_per_unit(tiles)
+        try:
+            outs.append(gpu_attn(q, k, v, n))
+        finally:
+            Bn.dlm_set_attn_tiles_per_unit(0)
+    assert torch.equal(outs[0], outs[1])
+

@@ -111,3 +111,26 @@ def test_full_size_sampled(mode):
         ref = oracle.bidir_attn(qs[None], ks[None], vs[None], [sl[b]], mask_mode=mode, block=64, prompt_lens=[pl[b]])
         err = np.abs(out[b, :, h] - ref[0, :, 0])
         assert err.max() <= ATTN_TOL_BF16, f"mode {mode} b {b} h {h}: {err.max()}"
+
+
+@pytest.mark.parametrize("mode", [CAUSAL, LOCAL])
+def test_workload_full_size(mode):
+    """The 32 x 512 workload with its prompt lengths under both block masks (64-token
+    blocks, the bench's setting): the whole batch in one launch, the oracle on
+    sampled (sequence, query head) pairs from host-generated inputs."""
+    from paper_2608_02625_gb300 import synth, synth_gpu
+    w = workloads.get("c3_batch32_512")
+    q, k, v = synth_gpu.qkv(w, 0, dev())
+    n, pl = w.seq_lens(), w.prompt_lens()
+    out = gpu_masked(q, k, v, n, pl, mode, 64)
+    g_out = out.float()
+    for b, heads in ((0, (0, 31)), (9, (5,)), (22, (13, 26)), (31, (7,))):
+        hq = host_qkv_seq(w, 0, synth.S_Q, b, w.Hq)
+        hk = host_qkv_seq(w, 0, synth.S_K, b, w.Hkv)
+        hv = host_qkv_seq(w, 0, synth.S_V, b, w.Hkv)
+        for h in heads:
+            g = (h * w.Hkv) // w.Hq
+            ref = oracle.bidir_attn(hq[None, :, h:h + 1], hk[None, :, g:g + 1], hv[None, :, g:g + 1], [n[b]],
+                                    mask_mode=mode, block=64, prompt_lens=[pl[b]])
+            compare(g_out[b:b + 1, :, h:h + 1], ref, [n[b]], ATTN_TOL_BF16, where=f"c3 mode {mode} b={b} h={h}")
+
